@@ -1,0 +1,139 @@
+"""CPU oracle for the WHTMix token mixer -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline / reference legs may
+import this package.  The product path (the C-ABI library and its Python binding) never does.
+
+The arithmetic lives in ``whtmix_oracle.c`` (plain C, float64 / uint32, single-threaded); this
+module only compiles it with gcc and marshals numpy arrays.  See the C file's header for what is
+computed and which passage of the paper (Section III-B, Eq. 1-4) each step follows.
+
+Every function here is pinned by ``tests/test_oracle.py`` against dense Sylvester-Hadamard
+products built independently (popcount definition, Sylvester recursion, scipy.linalg.hadamard),
+closed forms (delta inputs, single-frequency gains, unit gains), invariants (self-inverse,
+Parseval, linearity, adjointness) and finite differences.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "whtmix_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (-O2, no fast-math: IEEE float64 as written)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", "-std=c11", "-O2", "-fno-fast-math", "-ffp-contract=off", "-fPIC",
+                        "-shared", "-o", tmp, _SRC], check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            i64, p = ctypes.c_int64, ctypes.c_void_p
+            for name in ("oracle_fwht_f64", "oracle_fwht_u32"):
+                getattr(lib, name).argtypes = [p, i64, i64]
+                getattr(lib, name).restype = None
+            lib.oracle_wht2d_f64.argtypes = [p, p, i64, i64, i64]
+            for name in ("oracle_forward_f64", "oracle_forward_u32"):
+                getattr(lib, name).argtypes = [p, p, p, i64, i64, i64]
+            for name in ("oracle_backward_f64", "oracle_backward_u32"):
+                getattr(lib, name).argtypes = [p, p, p, p, p, i64, i64, i64]
+            for name in ("oracle_wht2d_f64", "oracle_forward_f64", "oracle_forward_u32",
+                         "oracle_backward_f64", "oracle_backward_u32"):
+                getattr(lib, name).restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _shape3(x: np.ndarray):
+    if x.ndim == 2:
+        return 1, x.shape[0], x.shape[1]
+    if x.ndim != 3:
+        raise ValueError("x must be [N, C] or [B, N, C]")
+    return x.shape
+
+
+def _check(rc: int):
+    if rc != 0:
+        raise ValueError(f"oracle error {rc} (N and C must be powers of two)")
+
+
+def fwht(v: np.ndarray) -> np.ndarray:
+    """Unnormalised FWHT of a 1D vector (float64, or uint32 with wrap-around)."""
+    lib = _load()
+    if v.dtype == np.uint32:
+        out = np.ascontiguousarray(v, dtype=np.uint32).copy()
+        lib.oracle_fwht_u32(_ptr(out), out.size, 1)
+    else:
+        out = np.ascontiguousarray(v, dtype=np.float64).copy()
+        lib.oracle_fwht_f64(_ptr(out), out.size, 1)
+    return out
+
+
+def wht2d(x: np.ndarray) -> np.ndarray:
+    """H_N X_b H_C for each plane (float64, unnormalised)."""
+    lib = _load()
+    B, N, C = _shape3(x)
+    xx = np.ascontiguousarray(x, dtype=np.float64)
+    out = np.empty_like(xx)
+    _check(lib.oracle_wht2d_f64(_ptr(xx), _ptr(out), B, N, C))
+    return out
+
+
+def forward(x: np.ndarray, g: np.ndarray) -> np.ndarray:
+    """WHTMix forward.  float inputs -> float64 orthonormal map; int32/uint32 -> integer mode
+    (unnormalised, mod 2^32) returned as int32."""
+    lib = _load()
+    B, N, C = _shape3(x)
+    if np.issubdtype(x.dtype, np.integer):
+        xx = np.ascontiguousarray(x).astype(np.uint32)
+        gg = np.ascontiguousarray(g).astype(np.uint32)
+        y = np.empty_like(xx)
+        _check(lib.oracle_forward_u32(_ptr(xx), _ptr(gg), _ptr(y), B, N, C))
+        return y.view(np.int32).reshape(x.shape)
+    xx = np.ascontiguousarray(x, dtype=np.float64)
+    gg = np.ascontiguousarray(g, dtype=np.float64)
+    y = np.empty_like(xx)
+    _check(lib.oracle_forward_f64(_ptr(xx), _ptr(gg), _ptr(y), B, N, C))
+    return y.reshape(x.shape)
+
+
+def backward(x: np.ndarray, g: np.ndarray, dy: np.ndarray):
+    """WHTMix backward: returns (dX, dG) with dG summed over the batch in ascending order."""
+    lib = _load()
+    B, N, C = _shape3(x)
+    if np.issubdtype(x.dtype, np.integer):
+        xx = np.ascontiguousarray(x).astype(np.uint32)
+        gg = np.ascontiguousarray(g).astype(np.uint32)
+        dd = np.ascontiguousarray(dy).astype(np.uint32)
+        dx = np.empty_like(xx)
+        dg = np.empty((N, C), dtype=np.uint32)
+        _check(lib.oracle_backward_u32(_ptr(xx), _ptr(gg), _ptr(dd), _ptr(dx), _ptr(dg), B, N, C))
+        return dx.view(np.int32).reshape(x.shape), dg.view(np.int32)
+    xx = np.ascontiguousarray(x, dtype=np.float64)
+    gg = np.ascontiguousarray(g, dtype=np.float64)
+    dd = np.ascontiguousarray(dy, dtype=np.float64)
+    dx = np.empty_like(xx)
+    dg = np.empty((N, C), dtype=np.float64)
+    _check(lib.oracle_backward_f64(_ptr(xx), _ptr(gg), _ptr(dd), _ptr(dx), _ptr(dg), B, N, C))
+    return dx.reshape(x.shape), dg
