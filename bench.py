@@ -1,0 +1,365 @@
+"""WHTMix forward benchmark: tokens/s and achieved HBM GB/s against the measured GB300 peak.
+
+One step = one whtmix_forward call (the whole hot path: load, forward 2D WHT, gain, inverse 2D
+WHT, store) over one batch of synthetic input already resident in HBM.  Default workload: the
+full-image global-mixing shape, X [1, 65536, 128] bf16 (two 135x240 maps flattened, zero-padded
+to 65536 tokens), G [65536, 128] fp32.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+
+Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs its own copy of the
+workload (independent planes, no collective on the data path: weak scaling); the timed region is
+bracketed by a barrier and a device synchronisation on both sides and the MAX over ranks is used.
+
+Timing: CUDA events on the stream the kernels run on.  The inputs rotate over enough buffer sets
+that their total exceeds 3x the L2 size, so every step streams X and G from HBM.  Clocks and
+throttle reasons are sampled with nvidia-smi during the run.  ``--impl reference`` times the CPU
+oracle (float64, single-threaded) on the host as the reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_25234_gb300 import inputs  # noqa: E402
+
+DEFAULT_WORKLOAD = "fullimage_1x65536x128_bf16"
+NOMINAL_HBM_GBS = 7900.0
+FALLBACK_HBM_GBS = 6800.0
+REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
+           0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+           0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_25234_gb300", "csrc", f) for f in
+                  ("whtmix_kernels.cuh", "whtmix_capi.cu")]
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in sorted(KERNEL_SOURCES):
+        if os.path.exists(f):
+            h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+class ClockSampler:
+    """nvidia-smi samples (timestamped on the host) for one GPU while the bench runs."""
+
+    def __init__(self, gpu_index: str):
+        self.samples = []  # (host_time, sm_mhz, max_mhz, reasons_mask)
+        self.proc = None
+        self.gpu = gpu_index
+        self._t = None
+
+    def start(self):
+        cmd = ["nvidia-smi", "-i", self.gpu, "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
+               "--format=csv,noheader,nounits", "-lms", "50"]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self._t = threading.Thread(target=self._read, daemon=True)
+        self._t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 3:
+                continue
+            try:
+                self.samples.append((time.time(), float(parts[0]), float(parts[1]), int(parts[2], 16)))
+            except ValueError:
+                pass
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+        if self._t is not None:
+            self._t.join(timeout=5)
+
+    def summary(self, t0: float, t1: float):
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        window = "timed_region"
+        if not inside:
+            inside, window = self.samples, "whole_run"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "window": "none"}
+        mask = 0
+        for s in inside:
+            mask |= s[3]
+        return {"sm_mhz": statistics.median(s[1] for s in inside), "sm_max_mhz": max(s[2] for s in inside),
+                "reasons": [n for b, n in REASONS.items() if mask & b and n != "gpu_idle"],
+                "samples": len(inside), "window": window}
+
+
+def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
+    """Median wall time of the CPU oracle's forward on one [n_tokens, C] plane of the workload."""
+    import numpy as np
+    import oracle
+    d = inputs.make_inputs(1, n_tokens, w.C, w.dtype, seed=0,
+                           n_valid=None if w.n_valid is None else min(w.n_valid, n_tokens))
+    x = inputs.as_float64(d["x"], w.dtype)
+    g = d["g"].astype(np.float64)
+    oracle.forward(x[:, :8, :], g[:8, :])  # load / compile outside the timing
+    times = []
+    for _ in range(reps):
+        t = time.perf_counter()
+        oracle.forward(x, g)
+        times.append(time.perf_counter() - t)
+    return statistics.median(times), times
+
+
+def reference_arm(args, w):
+    """The CPU oracle as the reference arm: each step runs the oracle forward on a bounded sample
+    (one plane; the full [N, C] plane when K+W steps of it fit in about three minutes, else a
+    plane with fewer tokens) and the metric is tokens/s of that sample."""
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle
+    t_full, _ = oracle_time_plane(w, w.N, 1)
+    budget = 180.0
+    n = w.N
+    while n > 64 and (args.steps + args.warmup) * t_full * n / w.N > budget:
+        n //= 2
+    d = inputs.make_inputs(1, n, w.C, w.dtype, seed=0, n_valid=None if w.n_valid is None else min(w.n_valid, n))
+    x = inputs.as_float64(d["x"], w.dtype)
+    g = d["g"].astype(np.float64)
+    for _ in range(args.warmup):
+        oracle.forward(x, g)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.forward(x, g)
+    el = time.perf_counter() - t0
+    value = args.steps * n / el
+    sample = f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s)"
+    line = {"impl": "reference", "metric": "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * el / max(args.steps, 1), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def traffic_from_profile(workload: str):
+    """dram bytes per launch from a committed ncu summary, only while the kernel sources match."""
+    p = os.path.join(ROOT, "profiles", "roofline_traffic.json")
+    try:
+        d = json.load(open(p))
+    except Exception:
+        return None
+    e = d.get(workload)
+    if not e or e.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def ours(args, w):
+    import ctypes
+    import numpy as np
+    import torch
+    from paper_2607_25234_gb300 import whtmix
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    lib = whtmix.library()
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 132 * 2**20
+
+    d = inputs.workload_inputs(w, seed=rank)
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16, "i32": torch.int32}[w.dtype]
+    x_host = torch.from_numpy(d["x"].view(np.int16) if w.dtype == "bf16" else d["x"])
+    if w.dtype == "bf16":
+        x_host = x_host.view(torch.bfloat16)
+    g_host = torch.from_numpy(d["g"])
+    x0 = x_host.to(dev)
+    g0 = g_host.to(dev)
+    set_bytes = x0.numel() * x0.element_size() * 2 + g0.numel() * g0.element_size()
+    nsets = max(2, -(-3 * l2 // set_bytes))
+    xs = [x0] + [x0.clone() for _ in range(nsets - 1)]
+    gs = [g0] + [g0.clone() for _ in range(nsets - 1)]
+    ys = [torch.empty_like(x0) for _ in range(nsets)]
+    code = whtmix.DTYPE_CODE[tdt]
+    stream = torch.cuda.current_stream(dev)
+    sp = int(stream.cuda_stream)
+    args_c = [(xs[i].data_ptr(), gs[i].data_ptr(), ys[i].data_ptr()) for i in range(nsets)]
+    fwd = lib.whtmix_forward
+
+    def step(i):
+        a = args_c[i % nsets]
+        rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
+        if rc != 0:
+            raise whtmix.WhtmixError(rc, "whtmix_forward")
+
+    # warm-up (also allocates the cached workspace on this stream)
+    for i in range(max(args.warmup, 3)):
+        step(i)
+    whtmix.sync(stream)
+
+    gpu_index = os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local if world > 1 and
+                                                                          "CUDA_VISIBLE_DEVICES" in os.environ else 0]
+    sampler = ClockSampler(gpu_index if "CUDA_VISIBLE_DEVICES" in os.environ else str(local))
+    sampler.start()
+    time.sleep(0.3)
+    for i in range(max(args.warmup, 3)):
+        step(i)
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_host0 = time.time()
+    start.record(stream)
+    for i in range(K):
+        ev[i][0].record(stream)
+        step(i)
+        ev[i][1].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    t_host1 = time.time()
+    if world > 1:
+        dist.barrier()
+    rc = lib.whtmix_sync(ctypes.c_void_p(sp))
+    if rc != 0:
+        raise whtmix.WhtmixError(rc, "device-side check after the timed loop")
+    elapsed_ms = start.elapsed_time(end)
+    kern_ms = [a.elapsed_time(b) for a, b in ev]
+    time.sleep(0.2)
+    sampler.stop()
+    clocks = sampler.summary(t_host0, t_host1)
+
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = t.item()
+
+    tokens_per_step = w.B * w.N
+    value = world * tokens_per_step * K / (elapsed_ms / 1e3)
+    kern_mean_ms = statistics.mean(kern_ms)
+    ideal = w.ideal_bytes(backward=False)
+    peak, peak_kind = measured_peaks()
+    achieved = ideal / (kern_mean_ms / 1e3) / 1e9
+
+    # end to end through the public Python API: pinned host buffers, copies inside the timed loop
+    e2e = None
+    if rank == 0 or world > 1:
+        xh = x_host.pin_memory()
+        gh = g_host.pin_memory()
+        yh = torch.empty_like(xh).pin_memory()
+        xd, gd, yd = xs[0], gs[0], ys[0]
+        ke = max(3, min(K, 50))
+        for _ in range(3):
+            xd.copy_(xh, non_blocking=True)
+            gd.copy_(gh, non_blocking=True)
+            whtmix.forward(xd, gd, out=yd)
+            yh.copy_(yd, non_blocking=True)
+        torch.cuda.synchronize(dev)
+        s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(ke):
+            xd.copy_(xh, non_blocking=True)
+            gd.copy_(gh, non_blocking=True)
+            whtmix.forward(xd, gd, out=yd)
+            yh.copy_(yd, non_blocking=True)
+        e2.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = s2.elapsed_time(e2) / ke
+        e2e = {"value": tokens_per_step / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": xh.numel() * xh.element_size() + gh.numel() * gh.element_size(),
+               "d2h_bytes_per_step": yh.numel() * yh.element_size(), "steps": ke, "ms_per_step": e2e_ms}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        t_med, times = oracle_time_plane(w, w.N, 3)
+        cpu = {"value": w.B * w.N / (t_med * w.B), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"one full [{w.N},{w.C}] plane of the workload (B={w.B} planes would take "
+                         f"{w.B * t_med:.2f} s), float64 oracle, median of 3 runs: "
+                         + ", ".join(f"{t:.2f}" for t in times) + " s"}
+
+    line = {"metric": "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
+                       "f32" if w.dtype != "i32" else "i32", "parallelism": f"replicas{world}",
+                       "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / 2**20:.0f} MiB, "
+                             f"{nsets * set_bytes / l2:.1f}x L2)"},
+            "hbm_gbs": achieved, "pct_of_measured_peak": 100.0 * achieved / peak,
+            "pct_of_nominal_peak": 100.0 * achieved / NOMINAL_HBM_GBS,
+            "kernel_us": {"mean": 1e3 * kern_mean_ms, "median": 1e3 * statistics.median(kern_ms),
+                          "p10": 1e3 * sorted(kern_ms)[len(kern_ms) // 10],
+                          "p90": 1e3 * sorted(kern_ms)[(9 * len(kern_ms)) // 10]},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic_from_profile(w.name),
+                         "peak_kind": peak_kind, "algorithmic_bytes_per_launch": ideal,
+                         "kernel": "whtmix k_forward_m (one launch per step)"},
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K, "clocks": clocks}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=inputs.WORKLOAD_ORDER)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    w = inputs.WORKLOADS[args.workload]
+    if w.backward:
+        raise SystemExit("the bench times the forward; the training-step workload is a parity case")
+    if args.impl == "reference":
+        reference_arm(args, w)
+    else:
+        ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

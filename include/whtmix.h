@@ -1,0 +1,138 @@
+/*
+ * whtmix.h -- C ABI of the WHTMix token mixer for NVIDIA GB300 (sm_103a).
+ *
+ * The operation (paper Section III-B, Eq. 1-4, "Walsh-Hadamard Token Mixer"): for each plane
+ * X_b [N, C] of a batch (tokens x channels) and one gain matrix G [N, C],
+ *
+ *     Y_b = H_N ( G (.) (H_N X_b H_C) ) H_C / (N C)
+ *
+ * where H_n is the n x n Sylvester-Hadamard matrix, (H_n)_{ij} = (-1)^{popcount(i & j)}.  With the
+ * orthonormal transform W = H_N (.) H_C / sqrt(N C) this is Y = W (G (.) W X): a forward 2D
+ * Walsh-Hadamard transform, a per-frequency gain, and the inverse transform (W is its own
+ * inverse).  The paper's learnable log-domain gains g_c, g_t are the rank-1 case
+ * G = exp(g_t) exp(g_c)^T; the input/output projections W_in, W_out (Eq. 1, Eq. 4) are dense
+ * GEMMs outside this call.  The paper zero-pads the token axis to a power of two before the
+ * transform; here N and C must already be powers of two (pad on the caller's side).
+ *
+ * The backward (not printed in the paper, which trains the block end to end; it follows from
+ * the map being linear in X and in G and from W being symmetric):
+ *
+ *     dX_b = H_N ( G (.) (H_N dY_b H_C) ) H_C / (N C)
+ *     dG   = sum_{b = 0 .. B-1, ascending} (H_N X_b H_C) (.) (H_N dY_b H_C) / (N C)
+ *
+ * Conventions for every call below
+ *   Layout      X, Y, dY, dX: row-major contiguous [B, N, C] (c fastest, then n, then b).
+ *               G, dG: row-major contiguous [N, C].  All are DEVICE pointers unless stated.
+ *   dtype       WHTMIX_F32:  X/Y/dY/dX float32, G/dG float32, orthonormal (1/(N C)), fp32 math.
+ *               WHTMIX_BF16: X/Y/dY/dX bfloat16, G/dG float32, orthonormal, fp32 math, the
+ *                            outputs rounded to nearest-even once at the store.
+ *               WHTMIX_I32:  X/Y/dY/dX int32, G/dG int32, UNnormalised (no 1/(N C)), every
+ *                            operation wraps modulo 2^32 -- the result is exact and independent
+ *                            of the order of the butterfly stages.
+ *   Shapes      B >= 0, N >= 1 and C >= 1 powers of two, N*C <= 2^26 elements per plane,
+ *               B*N*C < 2^62.  B = 0: the forward returns WHTMIX_OK without touching anything
+ *               (null data pointers are accepted); the backward sets dG to zero (the sum over no
+ *               planes) and touches nothing else, so only dgains must be valid.
+ *   Alignment   every pointer must be 16-byte aligned.
+ *   Aliasing    y == x (and dx == dy) is allowed and computes in place.  Any other overlap
+ *               between an output and an input or another output returns WHTMIX_ERR_ALIAS.
+ *   Streams     `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls are
+ *               asynchronous on that stream; all argument checks run on the host before anything
+ *               is enqueued, and a call that returns an error has enqueued nothing and written
+ *               nothing.  Faults of the device code surface at the caller's next synchronisation.
+ *   Ownership   the caller owns every pointer it passes.  The plain calls keep a workspace per
+ *               (device, stream), allocated stream-ordered on first use and grown on demand;
+ *               whtmix_release_workspaces() frees them.  The _ex calls use the caller's workspace
+ *               instead and allocate nothing.
+ *   Threads     calls on different streams may run concurrently from different host threads.
+ *               Two calls that share a workspace (same stream, or the same _ex buffer) must be
+ *               ordered by that stream.
+ */
+#ifndef WHTMIX_H
+#define WHTMIX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define WHTMIX_API __attribute__((visibility("default")))
+#else
+#define WHTMIX_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { WHTMIX_F32 = 0, WHTMIX_BF16 = 1, WHTMIX_I32 = 2 } whtmix_dtype_t;
+
+typedef enum {
+    WHTMIX_OK = 0,
+    WHTMIX_ERR_INVALID_ARG = 1, /* null pointer where data is needed, B < 0, N < 1 or C < 1   */
+    WHTMIX_ERR_BAD_SHAPE = 2,   /* N or C not a power of two, N*C > 2^26, B*N*C too large     */
+    WHTMIX_ERR_BAD_DTYPE = 3,   /* dtype not one of whtmix_dtype_t                             */
+    WHTMIX_ERR_MISALIGNED = 4,  /* a pointer is not 16-byte aligned                            */
+    WHTMIX_ERR_ALIAS = 5,       /* partial overlap between an output and another buffer        */
+    WHTMIX_ERR_CUDA = 6,        /* a CUDA runtime call failed: see whtmix_last_cuda_error()    */
+    WHTMIX_ERR_TIMEOUT = 7,     /* a bounded device-side wait expired (reported by whtmix_sync) */
+    WHTMIX_ERR_NO_DEVICE = 8,   /* no CUDA device, or the current device is not sm_103         */
+    WHTMIX_ERR_WORKSPACE = 9    /* _ex call: workspace null, misaligned or smaller than needed */
+} whtmix_status_t;
+
+/* Forward mixer.  Section III-B, Eq. 1-4 (the map between W_in and W_out).
+ *   x      [B, N, C] input planes (dtype)            gains  [N, C] G (float32, int32 for I32)
+ *   y      [B, N, C] output planes (dtype); may equal x.
+ * Returns a whtmix_status_t.  One kernel launch on `stream` (two for some shapes; none when
+ * B = 0). */
+WHTMIX_API int whtmix_forward(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
+                   int dtype, void *stream);
+
+/* Backward mixer: both gradients of the forward map.
+ *   x      [B, N, C] the forward input              gains [N, C] G
+ *   dy     [B, N, C] upstream gradient dL/dY          dx   [B, N, C] dL/dX (may equal dy)
+ *   dgains [N, C] dL/dG, float32 (int32 for I32), OVERWRITTEN (not accumulated into); the sum
+ *          over b runs in ascending b, so the result is bit-reproducible run to run.
+ * dgains may not overlap x, dy, dx or gains. */
+WHTMIX_API int whtmix_backward(const void *x, const void *gains, const void *dy, void *dx, void *dgains,
+                    int64_t B, int64_t N, int64_t C, int dtype, void *stream);
+
+/* Workspace size in bytes for the _ex calls (backward != 0 for whtmix_backward_ex).  Writes
+ * *out_bytes; the size depends only on the arguments. */
+WHTMIX_API int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype, int backward, size_t *out_bytes);
+
+/* Same as whtmix_forward / whtmix_backward with a caller-owned device workspace of at least
+ * whtmix_workspace_bytes() bytes, 256-byte aligned.  Its first 256 bytes hold a device-wide
+ * barrier (an arrival count, a generation word and an error word) and must be zero before the
+ * first call that uses the buffer (cudaMemset); every call that completes leaves the count and
+ * the error word zero (the generation word keeps advancing, which is harmless).  Calls sharing
+ * a workspace must be ordered on one stream. */
+WHTMIX_API int whtmix_forward_ex(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
+                      int dtype, void *workspace, size_t workspace_bytes, void *stream);
+WHTMIX_API int whtmix_backward_ex(const void *x, const void *gains, const void *dy, void *dx, void *dgains,
+                       int64_t B, int64_t N, int64_t C, int dtype, void *workspace,
+                       size_t workspace_bytes, void *stream);
+
+/* Synchronises `stream` and reports device-side failures of the calls enqueued on it since the
+ * previous whtmix_sync: WHTMIX_ERR_TIMEOUT if a bounded device-wide wait gave up (the library
+ * then resets that workspace's barrier), WHTMIX_ERR_CUDA if the synchronisation itself failed,
+ * WHTMIX_OK otherwise.  Only the library-managed workspaces of `stream` are checked. */
+WHTMIX_API int whtmix_sync(void *stream);
+
+/* Frees every library-managed workspace on the current device (synchronises the device). */
+WHTMIX_API int whtmix_release_workspaces(void);
+
+/* Static description of a status code; never NULL. */
+WHTMIX_API const char *whtmix_status_string(int status);
+
+/* The cudaError_t of the last CUDA failure seen by this host thread (0 if none). */
+WHTMIX_API int whtmix_last_cuda_error(void);
+
+/* Which kernel plan a shape uses: 1 = one tile per plane group (N*C <= 2^13), 2 = three
+ * passes through the workspace (2^13 < N*C <= 2^26); 0 for an invalid shape. */
+WHTMIX_API int whtmix_plan(int64_t N, int64_t C);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WHTMIX_H */

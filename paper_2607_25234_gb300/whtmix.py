@@ -1,0 +1,197 @@
+"""Python binding of the WHTMix C ABI (``include/whtmix.h``): argument marshalling only.
+
+Every step of the mixer runs in the CUDA library ``_lib/libwhtmix.so``; this module passes device
+pointers, sizes and the current CUDA stream through ctypes.  torch supplies device memory and
+streams.  There is no CPU path: a missing library or a CPU tensor raises.
+
+The operation (paper Section III-B, Eq. 1-4): Y_b = H_N (G (.) H_N X_b H_C) H_C / (N C) for every
+plane X_b [N, C] of X [B, N, C]; the backward returns dX and dG = sum_b (H X_b H)(H dY_b H)/(N C).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+__all__ = ["forward", "backward", "forward_ex", "backward_ex", "workspace_bytes", "sync", "plan",
+           "release_workspaces", "WhtmixError", "WHTMixFunction", "pad_tokens", "EXPORTS", "library"]
+
+# status codes and dtype codes of include/whtmix.h
+OK = 0
+STATUS = {0: "OK", 1: "INVALID_ARG", 2: "BAD_SHAPE", 3: "BAD_DTYPE", 4: "MISALIGNED", 5: "ALIAS",
+          6: "CUDA", 7: "TIMEOUT", 8: "NO_DEVICE", 9: "WORKSPACE"}
+DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.int32: 2}
+GAIN_DTYPE = {torch.float32: torch.float32, torch.bfloat16: torch.float32, torch.int32: torch.int32}
+
+# every entry point include/whtmix.h declares
+EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmix_forward_ex",
+           "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
+           "whtmix_last_cuda_error", "whtmix_plan")
+
+
+class WhtmixError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: WHTMIX_{'ERR_' if status else ''}{STATUS.get(status, status)} ({status})")
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library(path: str | None = None) -> ctypes.CDLL:
+    """Load the C library (built by ``__graft_entry__.build()``); raises if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = path or _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"WHTMix CUDA library not built ({path}); run __graft_entry__.build()")
+            lib = ctypes.CDLL(path)
+            i64, p, i, sz = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+            lib.whtmix_forward.argtypes = [p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_backward.argtypes = [p, p, p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_forward_ex.argtypes = [p, p, p, i64, i64, i64, i, p, sz, p]
+            lib.whtmix_backward_ex.argtypes = [p, p, p, p, p, i64, i64, i64, i, p, sz, p]
+            lib.whtmix_workspace_bytes.argtypes = [i64, i64, i64, i, i, ctypes.POINTER(sz)]
+            lib.whtmix_sync.argtypes = [p]
+            lib.whtmix_release_workspaces.argtypes = []
+            lib.whtmix_status_string.argtypes = [i]
+            lib.whtmix_status_string.restype = ctypes.c_char_p
+            lib.whtmix_last_cuda_error.argtypes = []
+            lib.whtmix_plan.argtypes = [i64, i64]
+            for name in EXPORTS:
+                if name != "whtmix_status_string":
+                    getattr(lib, name).restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _check(rc: int, what: str):
+    if rc != OK:
+        if rc == 6:
+            what += f" (cudaError {library().whtmix_last_cuda_error()})"
+        raise WhtmixError(rc, what)
+
+
+def _stream_ptr(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _shape(x: torch.Tensor):
+    if x.dim() == 2:
+        return 1, x.shape[0], x.shape[1]
+    if x.dim() != 3:
+        raise ValueError("x must be [N, C] or [B, N, C]")
+    return tuple(x.shape)
+
+
+def _check_tensors(x: torch.Tensor, g: torch.Tensor, *others: torch.Tensor):
+    if x.dtype not in DTYPE_CODE:
+        raise TypeError(f"unsupported dtype {x.dtype}; expected float32, bfloat16 or int32")
+    B, N, C = _shape(x)
+    if g.dtype != GAIN_DTYPE[x.dtype]:
+        raise TypeError(f"gains must be {GAIN_DTYPE[x.dtype]} for {x.dtype} inputs")
+    if tuple(g.shape) != (N, C):
+        raise ValueError(f"gains must be [N, C] = [{N}, {C}], got {tuple(g.shape)}")
+    for t in (x, g) + others:
+        if not t.is_cuda:
+            raise ValueError("WHTMix runs on CUDA tensors only")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    return B, N, C
+
+
+def forward(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Y = H_N (G (.) H_N X H_C) H_C / (N C) per plane (unnormalised, mod 2^32, for int32)."""
+    B, N, C = _check_tensors(x, g)
+    y = torch.empty_like(x) if out is None else out
+    if y.shape != x.shape or y.dtype != x.dtype:
+        raise ValueError("out must match x in shape and dtype")
+    _check(library().whtmix_forward(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype],
+                                    _stream_ptr(stream)), "whtmix_forward")
+    return y
+
+
+def backward(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torch.Tensor | None = None,
+             dg: torch.Tensor | None = None, stream=None):
+    """(dX, dG) of the forward map; dG is summed over the batch in ascending order."""
+    B, N, C = _check_tensors(x, g, dy)
+    if dy.shape != x.shape or dy.dtype != x.dtype:
+        raise ValueError("dy must match x in shape and dtype")
+    dx = torch.empty_like(dy) if dx is None else dx
+    dg = torch.empty_like(g) if dg is None else dg
+    _check(library().whtmix_backward(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
+                                     B, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_backward")
+    return dx, dg
+
+
+def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool = False) -> int:
+    out = ctypes.c_size_t(0)
+    _check(library().whtmix_workspace_bytes(B, N, C, DTYPE_CODE[dtype], int(backward), ctypes.byref(out)),
+           "whtmix_workspace_bytes")
+    return out.value
+
+
+def forward_ex(x, g, workspace: torch.Tensor, out=None, stream=None):
+    B, N, C = _check_tensors(x, g, workspace)
+    y = torch.empty_like(x) if out is None else out
+    _check(library().whtmix_forward_ex(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype],
+                                       workspace.data_ptr(), workspace.numel() * workspace.element_size(),
+                                       _stream_ptr(stream)), "whtmix_forward_ex")
+    return y
+
+
+def backward_ex(x, g, dy, workspace: torch.Tensor, dx=None, dg=None, stream=None):
+    B, N, C = _check_tensors(x, g, dy, workspace)
+    dx = torch.empty_like(dy) if dx is None else dx
+    dg = torch.empty_like(g) if dg is None else dg
+    _check(library().whtmix_backward_ex(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
+                                        B, N, C, DTYPE_CODE[x.dtype], workspace.data_ptr(),
+                                        workspace.numel() * workspace.element_size(), _stream_ptr(stream)),
+           "whtmix_backward_ex")
+    return dx, dg
+
+
+def sync(stream=None) -> None:
+    """Synchronise the stream and raise if a device-side bounded wait expired."""
+    _check(library().whtmix_sync(_stream_ptr(stream)), "whtmix_sync")
+
+
+def release_workspaces() -> None:
+    _check(library().whtmix_release_workspaces(), "whtmix_release_workspaces")
+
+
+def plan(N: int, C: int) -> int:
+    return library().whtmix_plan(N, C)
+
+
+def pad_tokens(x: torch.Tensor, n_pad: int | None = None) -> torch.Tensor:
+    """Zero-pads the token axis (dim -2) to the next power of two, as the paper does before H_N
+    (Section III-B).  Crop the mixer's output back with ``y[..., :n, :]``."""
+    n = x.shape[-2]
+    target = n_pad or (1 << (n - 1).bit_length())
+    if target == n:
+        return x.contiguous()
+    pad = torch.zeros(*x.shape[:-2], target - n, x.shape[-1], dtype=x.dtype, device=x.device)
+    return torch.cat([x, pad], dim=-2).contiguous()
+
+
+class WHTMixFunction(torch.autograd.Function):
+    """autograd wrapper: forward and backward both run in the CUDA library."""
+
+    @staticmethod
+    def forward(ctx, x, g):
+        ctx.save_for_backward(x, g)
+        return forward(x.contiguous(), g.contiguous())
+
+    @staticmethod
+    def backward(ctx, dy):
+        x, g = ctx.saved_tensors
+        dx, dg = backward(x, g, dy.contiguous())
+        return dx, dg

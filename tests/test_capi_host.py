@@ -1,0 +1,132 @@
+"""C-ABI checks that need no GPU: the library loads, exports every entry point include/whtmix.h
+declares, and rejects bad arguments on the host before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_25234_gb300 import build as libbuild
+from paper_2607_25234_gb300 import whtmix
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "whtmix.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    libbuild.build()
+    return whtmix.library()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"WHTMIX_API\s+[\w\s\*]+?\b(whtmix_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    assert "whtmix_forward" in names and "whtmix_backward" in names
+    assert set(names) == set(whtmix.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+    out = os.popen(f"nm -D --defined-only {libbuild.LIB}").read()
+    exported = set(re.findall(r"\bT (whtmix_\w+)", out))
+    assert exported == set(declared_symbols()), exported ^ set(declared_symbols())
+
+
+def test_status_strings(lib):
+    for code in range(10):
+        assert lib.whtmix_status_string(code)
+    assert lib.whtmix_status_string(0) == b"ok"
+    assert lib.whtmix_status_string(12345) == b"unknown status"
+
+
+def test_plan_and_workspace_sizes(lib):
+    assert lib.whtmix_plan(256, 32) == 1      # 2^13 elements: one tile
+    assert lib.whtmix_plan(256, 64) == 2      # 2^14: three phases
+    assert lib.whtmix_plan(65536, 1024) == 2  # 2^26: largest plane
+    assert lib.whtmix_plan(65536, 2048) == 0  # 2^27: too large
+    assert lib.whtmix_plan(3, 4) == 0
+    ws = whtmix.workspace_bytes
+    import torch
+    assert ws(1, 256, 32, torch.float32) == 256
+    assert ws(1, 65536, 128, torch.bfloat16) == 256 + (1 << 23) * 4
+    # training step [16, 8192, 256]: forward groups of 4 planes, backward groups of 2 (two buffers)
+    assert ws(16, 8192, 256, torch.bfloat16) == 256 + 4 * (1 << 21) * 4
+    assert ws(16, 8192, 256, torch.bfloat16, backward=True) == 256 + 2 * 2 * (1 << 21) * 4
+    assert ws(0, 4, 4, torch.float32, backward=True) == 256 + 16 * 4
+
+
+FAKE = 1 << 20  # 16-byte aligned host integers posing as device pointers: never dereferenced
+
+
+def fwd(lib, x=FAKE, g=2 * FAKE, y=3 * FAKE, B=1, N=4, C=4, dtype=0):
+    return lib.whtmix_forward(x, g, y, B, N, C, dtype, None)
+
+
+def bwd(lib, x=FAKE, g=2 * FAKE, dy=3 * FAKE, dx=4 * FAKE, dg=5 * FAKE, B=1, N=4, C=4, dtype=0):
+    return lib.whtmix_backward(x, g, dy, dx, dg, B, N, C, dtype, None)
+
+
+def test_rejects_invalid_arguments_before_any_device_work(lib):
+    assert fwd(lib, x=None) == 1
+    assert fwd(lib, g=None) == 1
+    assert fwd(lib, y=None) == 1
+    assert fwd(lib, B=-1) == 1
+    assert fwd(lib, N=0) == 1
+    assert fwd(lib, C=0) == 1
+    assert fwd(lib, N=6) == 2
+    assert fwd(lib, C=12) == 2
+    assert fwd(lib, N=1 << 20, C=1 << 7) == 2
+    assert fwd(lib, dtype=3) == 3
+    assert fwd(lib, dtype=-1) == 3
+    assert fwd(lib, x=FAKE + 4) == 4
+    assert fwd(lib, y=3 * FAKE + 8) == 4
+    assert bwd(lib, dy=None) == 1
+    assert bwd(lib, dg=None) == 1
+    assert bwd(lib, dg=5 * FAKE + 2) == 4
+
+
+def test_alias_rules(lib):
+    n = 4 * 4 * 4  # bytes of a [1, 4, 4] f32 plane
+    assert fwd(lib, y=FAKE + 16) == 5                 # partial overlap with x
+    assert fwd(lib, y=2 * FAKE) == 5                  # output on top of the gains
+    assert bwd(lib, dx=3 * FAKE + 16) == 5            # partial overlap with dy
+    assert bwd(lib, dx=FAKE) == 5                     # dx over x
+    assert bwd(lib, dg=FAKE + 16) == 5                # dG inside x
+    assert bwd(lib, dg=4 * FAKE) == 5                 # dG over dx
+    assert bwd(lib, dg=2 * FAKE) == 5                 # dG over G
+    # exact in-place is allowed: with no GPU the call gets past every check and stops at the device
+    assert fwd(lib, y=FAKE) in (0, 6, 8)
+    assert bwd(lib, dx=3 * FAKE) in (0, 6, 8)
+    del n
+
+
+def test_empty_batch(lib):
+    assert fwd(lib, B=0) == 0
+    assert fwd(lib, x=None, g=None, y=None, B=0) == 0
+    assert bwd(lib, B=0, dg=None) == 1
+    assert bwd(lib, B=0, dg=5 * FAKE + 4) == 4
+    import torch
+    if not torch.cuda.is_available():
+        assert bwd(lib, x=None, dy=None, dx=None, B=0) == 8  # would zero dG on a GPU
+
+
+def test_ex_workspace_checks(lib):
+    f = lib.whtmix_forward_ex
+    need = ctypes.c_size_t(0)
+    assert lib.whtmix_workspace_bytes(1, 256, 64, 0, 0, ctypes.byref(need)) == 0
+    assert f(FAKE, 2 * FAKE, 3 * FAKE, 1, 256, 64, 0, None, need.value, None) == 9
+    assert f(FAKE, 2 * FAKE, 3 * FAKE, 1, 256, 64, 0, 8 * FAKE + 16, need.value, None) == 9
+    assert f(FAKE, 2 * FAKE, 3 * FAKE, 1, 256, 64, 0, 8 * FAKE, need.value - 1, None) == 9
+
+
+def test_no_device_reported_on_a_cpu_box(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    assert fwd(lib) == 8

@@ -1,0 +1,243 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 / uint32 CPU oracle on the same
+seeded inputs.
+
+Tolerances (per plane, Y_ref the fp64 oracle on the exact stored inputs):
+  int32      bit-exact (the integer mode is exact modulo 2^32 in any stage order);
+  float32    relative L2 <= 1e-6 and max abs <= 1e-5;
+  bfloat16   relative L2 <= 1e-2 (fp32 arithmetic, one rounding to bf16 at the store).
+dG is checked as one [N, C] plane with the same tolerance as its dtype's outputs.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_25234_gb300 import inputs, whtmix
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": (1e-6, 1e-5), "bf16": (1e-2, None)}
+TORCH_DT = {"f32": torch.float32, "bf16": torch.bfloat16, "i32": torch.int32}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2607_25234_gb300 import build
+    build.build()
+    oracle.build()
+    torch.cuda.set_device(0)
+
+
+def to_dev(a: np.ndarray, dtype: str) -> torch.Tensor:
+    if dtype == "bf16":
+        return torch.from_numpy(a.view(np.int16)).cuda().view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def to_f64(t: torch.Tensor) -> np.ndarray:
+    return t.double().cpu().numpy()
+
+
+def ref_inputs(d: dict, dtype: str):
+    """Exact float64 (or uint32) views of the stored inputs, as the GPU sees them."""
+    if dtype == "i32":
+        return {k: v for k, v in d.items()}
+    return {k: inputs.as_float64(v, dtype if k != "g" else "f32") for k, v in d.items()}
+
+
+def assert_close(got: torch.Tensor, ref: np.ndarray, dtype: str, what: str):
+    if dtype == "i32":
+        g = got.cpu().numpy().reshape(ref.shape)
+        assert np.array_equal(g, ref), f"{what}: {np.count_nonzero(g != ref)} of {g.size} int32 values differ"
+        return
+    rel_tol, abs_tol = TOL[dtype]
+    g = to_f64(got)
+    planes_g = g.reshape(-1, ref.shape[-2] * ref.shape[-1])
+    planes_r = ref.reshape(-1, ref.shape[-2] * ref.shape[-1])
+    for b in range(planes_r.shape[0]):
+        nr = np.linalg.norm(planes_r[b])
+        err = np.linalg.norm(planes_g[b] - planes_r[b])
+        assert err <= rel_tol * max(nr, 1e-30) or (nr == 0 and err == 0), \
+            f"{what} plane {b}: relative L2 {err / max(nr, 1e-30):.3e} > {rel_tol}"
+    if abs_tol is not None:
+        mx = np.abs(g - ref).max() if g.size else 0.0
+        assert mx <= abs_tol, f"{what}: max abs error {mx:.3e} > {abs_tol}"
+
+
+def run_forward(B, N, C, dtype, seed=0, n_valid=None):
+    d = inputs.make_inputs(B, N, C, dtype, seed=seed, n_valid=n_valid)
+    x, g = to_dev(d["x"], dtype), to_dev(d["g"], "f32" if dtype != "i32" else "i32")
+    y = whtmix.forward(x, g)
+    whtmix.sync()
+    r = ref_inputs(d, dtype)
+    y_ref = oracle.forward(r["x"], r["g"])
+    assert_close(y, y_ref, dtype, f"Y [{B},{N},{C}] {dtype}")
+    return x, g, y
+
+
+def run_backward(B, N, C, dtype, seed=0, n_valid=None):
+    d = inputs.make_inputs(B, N, C, dtype, seed=seed, n_valid=n_valid, with_dy=True)
+    gdt = "f32" if dtype != "i32" else "i32"
+    x, g, dy = to_dev(d["x"], dtype), to_dev(d["g"], gdt), to_dev(d["dy"], dtype)
+    dx, dg = whtmix.backward(x, g, dy)
+    whtmix.sync()
+    r = ref_inputs(d, dtype)
+    dx_ref, dg_ref = oracle.backward(r["x"], r["g"], r["dy"])
+    assert_close(dx, dx_ref, dtype, f"dX [{B},{N},{C}] {dtype}")
+    assert_close(dg, dg_ref[None], dtype if dtype == "i32" else "f32" if dtype == "f32" else "bf16",
+                 f"dG [{B},{N},{C}] {dtype}")
+    return dx, dg
+
+
+# ---- the five workloads at full size ----
+
+def test_tiny_1x256x64_f32_forward():
+    run_forward(1, 256, 64, "f32")
+
+
+def test_tiny_1x256x64_i32_forward_bit_exact():
+    run_forward(1, 256, 64, "i32")
+
+
+def test_epipolar_128x512x128_bf16_forward():
+    run_forward(128, 512, 128, "bf16")
+
+
+def test_longseq_32x4096x64_f32_forward():
+    run_forward(32, 4096, 64, "f32")
+
+
+def test_fullimage_1x65536x128_bf16_forward_padded():
+    run_forward(1, 65536, 128, "bf16", n_valid=2 * 135 * 240)
+
+
+def test_fullimage_1x65536x128_bf16_forward_dense():
+    run_forward(1, 65536, 128, "bf16")
+
+
+def test_train_16x8192x256_bf16_forward_backward():
+    run_forward(16, 8192, 256, "bf16")
+    run_backward(16, 8192, 256, "bf16")
+
+
+# ---- shape sweep: single-tile and three-phase plans, aspect ratios, ragged batches ----
+
+SWEEP = [(1, 1, 1), (3, 1, 1), (5, 1, 8), (7, 8, 1), (3, 2, 2), (9, 4, 16), (2, 16, 4), (33, 32, 8),
+         (3, 64, 128), (2, 128, 64), (1, 8192, 1), (1, 1, 8192), (2, 1, 16384), (3, 16384, 1),
+         (2, 64, 256), (3, 512, 32), (1, 2048, 64), (2, 256, 1024), (1, 1 << 18, 2), (1, 2, 1 << 18)]
+
+
+@pytest.mark.parametrize("B,N,C", SWEEP)
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "i32"])
+def test_forward_sweep(B, N, C, dtype):
+    run_forward(B, N, C, dtype, seed=B + N + C)
+
+
+@pytest.mark.parametrize("B,N,C", [(1, 1, 1), (3, 4, 2), (5, 32, 16), (2, 64, 128), (3, 128, 128),
+                                   (4, 1024, 64), (2, 8192, 2), (1, 1 << 17, 4), (6, 512, 16)])
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "i32"])
+def test_backward_sweep(B, N, C, dtype):
+    run_backward(B, N, C, dtype, seed=2 * B + N + C)
+
+
+def test_largest_plane_2_pow_26_bf16():
+    run_forward(1, 1 << 19, 128, "bf16", seed=3)
+
+
+def test_many_groups_forward_and_backward_f32():
+    # 2^20 elements per plane: forward groups of 8 planes, backward groups of 4
+    run_forward(20, 4096, 256, "f32", seed=4)
+    run_backward(10, 4096, 256, "f32", seed=5)
+
+
+# ---- semantics ----
+
+def test_integer_mode_wraps_mod_2_32():
+    B, N, C = 2, 512, 64
+    x = inputs.small_ints(80, B * N * C, -(2**31), 2**31 - 1).reshape(B, N, C)
+    g = inputs.small_ints(81, N * C, -(2**31), 2**31 - 1).reshape(N, C)
+    y = whtmix.forward(to_dev(x, "i32"), to_dev(g, "i32"))
+    assert np.array_equal(y.cpu().numpy(), oracle.forward(x, g))
+
+
+def test_in_place_forward_and_backward():
+    for (B, N, C) in [(3, 64, 64), (2, 1024, 128)]:
+        d = inputs.make_inputs(B, N, C, "f32", seed=6, with_dy=True)
+        x = to_dev(d["x"], "f32")
+        g = to_dev(d["g"], "f32")
+        y_ref = oracle.forward(d["x"].astype(np.float64), d["g"].astype(np.float64))
+        whtmix.forward(x, g, out=x)
+        assert_close(x, y_ref, "f32", "in-place Y")
+        dy = to_dev(d["dy"], "f32")
+        xx = to_dev(d["x"], "f32")
+        dx_ref, _ = oracle.backward(d["x"].astype(np.float64), d["g"].astype(np.float64), d["dy"].astype(np.float64))
+        whtmix.backward(xx, g, dy, dx=dy)
+        assert_close(dy, dx_ref, "f32", "in-place dX")
+
+
+def test_backward_is_deterministic():
+    d = inputs.make_inputs(8, 2048, 64, "bf16", seed=7, with_dy=True)
+    x, g, dy = to_dev(d["x"], "bf16"), to_dev(d["g"], "f32"), to_dev(d["dy"], "bf16")
+    a = whtmix.backward(x, g, dy)
+    b = whtmix.backward(x, g, dy)
+    torch.cuda.synchronize()
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+    d = inputs.make_inputs(40, 32, 16, "f32", seed=8, with_dy=True)
+    x, g, dy = to_dev(d["x"], "f32"), to_dev(d["g"], "f32"), to_dev(d["dy"], "f32")
+    a = whtmix.backward(x, g, dy)
+    b = whtmix.backward(x, g, dy)
+    torch.cuda.synchronize()
+    assert torch.equal(a[1], b[1])
+
+
+def test_unit_gain_is_identity_and_zero_gain_is_zero():
+    B, N, C = 2, 4096, 64
+    d = inputs.make_inputs(B, N, C, "f32", seed=9)
+    x = to_dev(d["x"], "f32")
+    y = whtmix.forward(x, torch.ones(N, C, device="cuda"))
+    assert (y - x).abs().max().item() <= 1e-5
+    y0 = whtmix.forward(x, torch.zeros(N, C, device="cuda"))
+    assert y0.abs().max().item() == 0.0
+
+
+def test_ex_variant_matches_plain_call():
+    B, N, C = 2, 8192, 32
+    d = inputs.make_inputs(B, N, C, "bf16", seed=10, with_dy=True)
+    x, g, dy = to_dev(d["x"], "bf16"), to_dev(d["g"], "f32"), to_dev(d["dy"], "bf16")
+    ws = torch.zeros(whtmix.workspace_bytes(B, N, C, torch.bfloat16, backward=True), dtype=torch.uint8, device="cuda")
+    y1 = whtmix.forward(x, g)
+    y2 = whtmix.forward_ex(x, g, ws)
+    dx1, dg1 = whtmix.backward(x, g, dy)
+    dx2, dg2 = whtmix.backward_ex(x, g, dy, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2) and torch.equal(dx1, dx2) and torch.equal(dg1, dg2)
+    header = ws[:256].view(torch.int32).cpu()
+    assert header[0].item() == 0 and header[2].item() == 0  # arrival count and error word back at zero
+
+
+def test_empty_batch_and_errors_on_gpu():
+    x = torch.empty(0, 16, 16, device="cuda")
+    g = torch.ones(16, 16, device="cuda")
+    y = whtmix.forward(x, g)
+    assert y.shape == (0, 16, 16)
+    dg = torch.full((16, 16), 7.0, device="cuda")
+    whtmix.backward(x, g, torch.empty_like(x), dg=dg)
+    torch.cuda.synchronize()
+    assert dg.abs().max().item() == 0.0  # the sum over an empty batch
+    with pytest.raises(whtmix.WhtmixError) as e:
+        whtmix.forward(torch.zeros(1, 12, 16, device="cuda"), torch.zeros(12, 16, device="cuda"))
+    assert e.value.status == 2
+    with pytest.raises(ValueError):
+        whtmix.forward(torch.zeros(1, 16, 16), torch.zeros(16, 16))
+
+
+def test_autograd_function():
+    B, N, C = 2, 256, 64
+    d = inputs.make_inputs(B, N, C, "f32", seed=11, with_dy=True)
+    x = to_dev(d["x"], "f32").requires_grad_(True)
+    g = to_dev(d["g"], "f32").requires_grad_(True)
+    y = whtmix.WHTMixFunction.apply(x, g)
+    y.backward(to_dev(d["dy"], "f32"))
+    dx_ref, dg_ref = oracle.backward(d["x"].astype(np.float64), d["g"].astype(np.float64), d["dy"].astype(np.float64))
+    assert_close(x.grad, dx_ref, "f32", "autograd dX")
+    assert_close(g.grad, dg_ref[None], "f32", "autograd dG")
