@@ -15,7 +15,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libwhtmix.so")
-SOURCES = ["whtmix_capi.cu"]
+SOURCES = ["whtmix_capi.cu", "whtmix_noalloc.cu"]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 

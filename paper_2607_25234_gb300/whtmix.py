@@ -30,7 +30,7 @@ GAIN_DTYPE = {torch.float32: torch.float32, torch.bfloat16: torch.float32, torch
 # every entry point include/whtmix.h declares
 EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmix_forward_ex",
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
-           "whtmix_last_cuda_error", "whtmix_plan")
+           "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc")
 
 
 class WhtmixError(RuntimeError):
