@@ -40,7 +40,15 @@ REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_c
            0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
            0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_25234_gb300", "csrc", f) for f in
-                  ("whtmix_kernels.cuh", "whtmix_capi.cu")]
+                  ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_capi.cu")]
+
+
+def kernel_name(w) -> str:
+    """The kernel one whtmix_forward call launches for this workload (mirrors the C ABI's dispatch)."""
+    m = (w.N * w.C).bit_length() - 1
+    if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
+        return f"k_forward_fast<{w.dtype}, Q={m - 13}>"
+    return "k_forward_s" if m <= 13 else "k_forward_m"
 
 
 def kernel_source_hash() -> str:
@@ -336,7 +344,7 @@ def ours(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic_from_profile(w.name),
                          "peak_kind": peak_kind, "algorithmic_bytes_per_launch": ideal,
-                         "kernel": "whtmix k_forward_m (one launch per step)"},
+                         "kernel": kernel_name(w) + " (one launch per step)"},
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K, "clocks": clocks}
     print(json.dumps(line), flush=True)
     if world > 1:

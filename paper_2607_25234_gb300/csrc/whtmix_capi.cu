@@ -12,6 +12,7 @@
 #include <utility>
 
 #include "whtmix.h"
+#include "whtmix_fast_launch.cuh"
 #include "whtmix_kernels.cuh"
 
 using namespace whtmix;
@@ -182,12 +183,23 @@ int launch(K kernel, bool cooperative, int sms, long long max_units, size_t smem
   return WHTMIX_OK;
 }
 
+// The fast forward (whtmix_fast.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^23.
+bool use_fast_forward(int dtype, int m) {
+  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m > fast::RB && m <= fast::RB + 10;
+}
+
 template <int D>
 int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
   using A = typename Tr<D>::A;
   const int m = P.m;
   const size_t tile_bytes = sizeof(A) * TILE;
   if (!backward) {
+    if constexpr (D != DT_I32) {
+      if (use_fast_forward(D, m)) {
+        const cudaError_t e = D == DT_BF16 ? fast::forward_bf16(P, sms, stream) : fast::forward_f32(P, sms, stream);
+        return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+      }
+    }
     if (m <= TILE_BITS) {
       const long long ppt = 1ll << (TILE_BITS - m);
       return launch(k_forward_s<D>, false, sms, (P.B + ppt - 1) / ppt, tile_bytes, P, stream);

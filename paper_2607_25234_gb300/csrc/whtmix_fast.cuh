@@ -1,0 +1,557 @@
+// whtmix_fast.cuh -- register/TMEM forward kernel for large planes (2^14 <= N*C <= 2^23), fp32 and
+// bf16 I/O.
+//
+// Same three phases as the generic plan M (Section III-B map; see whtmix_kernels.cuh), written
+// for the instruction and latency budget of the path: the butterflies need 2 log2(NC) fp32 adds
+// per element, which at N*C = 2^23 on 152 SMs is about as long as streaming X, G and Y through
+// HBM, and every SM must keep ~100 KB of loads in flight to hide memory latency.  So:
+//   * butterflies run on register pairs with packed add/sub.f32x2 (half the instructions);
+//   * one CTA of 8 warps per SM; phase 1 / phase 3 work on rows of 2^13 elements, one row per
+//     64-thread worker (4 per CTA), 128 elements per thread, exactly one shared-memory exchange
+//     per row (conflict-free XOR swizzle), on a balanced contiguous range of rows per SM;
+//   * phase 2 gives columns to threads: whole columns in registers when a column has <= 128
+//     elements; otherwise the two warps (w, w+4) that share a TMEM lane quarter hold one column
+//     per lane (Blackwell tensor memory as per-thread storage, 256 fp32 per thread), trade the
+//     bit between their halves through TMEM, and a 1024-element column adds one shuffle stage;
+//   * column ranges are balanced and aligned to 8 columns (32-byte sectors); G is prefetched into
+//     L2 during phase 1, which is bound by its writes and leaves HBM reads idle.
+// Phase 2's flat-index bits are the row bits [13, m); the gain multiplies by G[j*2^13 + c]/L.
+#pragma once
+
+#include "whtmix_kernels.cuh"
+
+namespace whtmix {
+namespace fast {
+
+constexpr int THREADS = 256;   // 8 warps: four 64-thread row workers; warps w, w+4 share TMEM lanes
+constexpr int RB = 13;         // row bits
+constexpr int ROWLEN = 1 << RB;
+constexpr int WORKER = 64;     // threads per row worker
+constexpr int NWORKERS = THREADS / WORKER;
+// four row exchange buffers (128 KiB): more than half an SM, so exactly one CTA runs per SM
+constexpr size_t SMEM_BYTES = NWORKERS * ROWLEN * sizeof(float);
+constexpr int G_PREFETCH_EIGHTHS = 8;  // share of G's rows (in eighths) prefetched into L2 in phase 1
+
+// ---------------------------------------------------------------------------------------------
+// packed fp32 pairs
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  float2 r;
+  asm("{.reg .b64 pa, pb, pd;\n\t"
+      "mov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+      "add.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;}"
+      : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+  float2 r;
+  asm("{.reg .b64 pa, pb, pd;\n\t"
+      "mov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+      "sub.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;}"
+      : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  float2 r;
+  asm("{.reg .b64 pa, pb, pd;\n\t"
+      "mov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+      "mul.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;}"
+      : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+// a * s + b with s = +-1 (exact)
+__device__ __forceinline__ float2 fma2(float2 a, float2 s, float2 b) {
+  float2 r;
+  asm("{.reg .b64 pa, ps, pb, pd;\n\t"
+      "mov.b64 pa, {%2, %3};\n\tmov.b64 ps, {%4, %5};\n\tmov.b64 pb, {%6, %7};\n\t"
+      "fma.rn.f32x2 pd, pa, ps, pb;\n\tmov.b64 {%0, %1}, pd;}"
+      : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(s.x), "f"(s.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+
+// butterfly on two pairs: (a, b) -> (a + b, a - b), elementwise
+__device__ __forceinline__ void bf2(float2& a, float2& b) {
+  const float2 s = add2(a, b), d = sub2(a, b);
+  a = s;
+  b = d;
+}
+// butterfly inside one pair: (x, y) -> (x + y, x - y)
+__device__ __forceinline__ void bf_in(float2& a) {
+  const float s = a.x + a.y, d = a.x - a.y;
+  a.x = s;
+  a.y = d;
+}
+
+// Butterflies over the bits of an index into v[]: for every h = 1, 2, ..., N/2 pair (i, i + h).
+template <int N>
+__device__ __forceinline__ void bfly_all(float2 (&v)[N]) {
+#pragma unroll
+  for (int h = 1; h < N; h <<= 1)
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+      if ((i & h) == 0) bf2(v[i], v[i + h]);
+}
+
+// ---------------------------------------------------------------------------------------------
+// TMEM (tensor memory) as per-thread storage: thread t of warp w owns lane 32*(w%4) + t.
+__device__ __forceinline__ void tmem_alloc_512(uint32_t* smem_slot) {
+  const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(smem_slot));
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(dst) : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_512(uint32_t taddr) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tmem_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// 16 consecutive 32-bit columns of this thread's lane <-> registers
+__device__ __forceinline__ void tmem_ld16(uint32_t ta, float (&r)[16]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+               : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]), "=f"(r[6]), "=f"(r[7]),
+                 "=f"(r[8]), "=f"(r[9]), "=f"(r[10]), "=f"(r[11]), "=f"(r[12]), "=f"(r[13]), "=f"(r[14]), "=f"(r[15])
+               : "r"(ta) : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t ta, const float (&r)[16]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+               ::"r"(ta), "f"(r[0]), "f"(r[1]), "f"(r[2]), "f"(r[3]), "f"(r[4]), "f"(r[5]), "f"(r[6]), "f"(r[7]),
+                 "f"(r[8]), "f"(r[9]), "f"(r[10]), "f"(r[11]), "f"(r[12]), "f"(r[13]), "f"(r[14]), "f"(r[15])
+               : "memory");
+}
+
+// ---------------------------------------------------------------------------------------------
+// Row exchange buffer: word address of row element r (13 bits), XOR-swizzled so that both access
+// patterns below are bank-conflict free:
+//   layout V (16-byte vectors of r0..r1, lanes on r3..r7): bits 2..4 = (r2^r5, r3^r9, r4^r10)
+//   layout P (8-byte pairs of r0, lanes on r1, r2, r9, r10, r11): bits 1..4 = (r1, r2^r5, r3^r9, r4^r10)
+__device__ __forceinline__ int xswz(int r) {
+  return r ^ (((r >> 5) & 1) << 2) ^ (((r >> 9) & 1) << 3) ^ (((r >> 10) & 1) << 4);
+}
+
+__device__ __forceinline__ void worker_sync(int worker) {
+  asm volatile("bar.sync %0, %1;" ::"r"(worker + 1), "r"(WORKER) : "memory");
+}
+
+// Storage <-> fp32 for the two floating dtypes.
+template <int D> struct IOv;
+template <> struct IOv<DT_BF16> {
+  // 8 consecutive elements at element index e (16-byte aligned): 4 pairs (r0 = 0, 1)
+  __device__ static __forceinline__ void ld8(const void* p, long long e, float2 (&o)[4]) {
+    const uint4 u = __ldcs(reinterpret_cast<const uint4*>(static_cast<const unsigned short*>(p) + e));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+  }
+  __device__ static __forceinline__ void st8(void* p, long long e, const float2 (&v)[4]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(v[i].x, v[i].y);
+      w[i] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    __stcs(reinterpret_cast<uint4*>(static_cast<unsigned short*>(p) + e), make_uint4(w[0], w[1], w[2], w[3]));
+  }
+};
+template <> struct IOv<DT_F32> {
+  __device__ static __forceinline__ void ld8(const void* p, long long e, float2 (&o)[4]) {
+    const float4* q = reinterpret_cast<const float4*>(static_cast<const float*>(p) + e);
+    const float4 a = __ldcs(q), b = __ldcs(q + 1);
+    o[0] = make_float2(a.x, a.y);
+    o[1] = make_float2(a.z, a.w);
+    o[2] = make_float2(b.x, b.y);
+    o[3] = make_float2(b.z, b.w);
+  }
+  __device__ static __forceinline__ void st8(void* p, long long e, const float2 (&v)[4]) {
+    float4* q = reinterpret_cast<float4*>(static_cast<float*>(p) + e);
+    __stcs(q, make_float4(v[0].x, v[0].y, v[1].x, v[1].y));
+    __stcs(q + 1, make_float4(v[2].x, v[2].y, v[3].x, v[3].y));
+  }
+};
+
+// ---------------------------------------------------------------------------------------------
+// Phase 1 row: X (dtype D) -> workspace (fp32), butterflies on all 13 row bits.
+//   layout V: thread wt holds r0..r2 (8-vectors) x r9..r12 (16 vectors); wt = r3..r8.
+//     round A: bits r1, r2, r9..r12 (pairs on r0).
+//   exchange through smem, then layout P: thread holds pairs (r0) x r3..r8; wt bits =
+//     (r1, r2, r9, r10, r11, r12).  round B: r0 (inside the pairs) and r3..r8.
+template <int D>
+__device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, int wt, int worker) {
+  float2 a[16][4];  // [v = r9..r12][r1 + 2 r2]
+#pragma unroll
+  for (int v = 0; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + 512 * v, a[v]);
+  // round A
+#pragma unroll
+  for (int v = 0; v < 16; ++v) {
+    bf2(a[v][0], a[v][1]);
+    bf2(a[v][2], a[v][3]);
+    bf2(a[v][0], a[v][2]);
+    bf2(a[v][1], a[v][3]);
+  }
+#pragma unroll
+  for (int h = 1; h < 16; h <<= 1)
+#pragma unroll
+    for (int v = 0; v < 16; ++v)
+      if ((v & h) == 0)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
+  // exchange V -> P
+#pragma unroll
+  for (int v = 0; v < 16; ++v)
+#pragma unroll
+    for (int r2 = 0; r2 < 2; ++r2) {
+      const int r = 8 * wt + 512 * v + 4 * r2;
+      *reinterpret_cast<float4*>(xbuf + xswz(r)) = make_float4(a[v][2 * r2].x, a[v][2 * r2].y, a[v][2 * r2 + 1].x, a[v][2 * r2 + 1].y);
+    }
+  worker_sync(worker);
+  const int pbase = 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2);  // r1, r2, r9..r12
+  float2 b[64];  // [s = r3..r8]
+#pragma unroll
+  for (int s = 0; s < 64; ++s) b[s] = *reinterpret_cast<const float2*>(xbuf + xswz(pbase + 8 * s));
+  worker_sync(worker);  // buffer free for the next row
+  // round B
+#pragma unroll
+  for (int s = 0; s < 64; ++s) bf_in(b[s]);
+  bfly_all<64>(b);
+#pragma unroll
+  for (int s = 0; s < 64; ++s) __stcg(reinterpret_cast<float2*>(dst_ws + pbase + 8 * s), b[s]);
+}
+
+// Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all 13 row bits (mirror of phase 1).
+template <int D>
+__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, float* xbuf, int wt, int worker) {
+  const int pbase = 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2);
+  float2 b[64];
+#pragma unroll
+  for (int s = 0; s < 64; ++s) b[s] = __ldcg(reinterpret_cast<const float2*>(src_ws + pbase + 8 * s));
+  bfly_all<64>(b);  // round A: r3..r8
+#pragma unroll
+  for (int s = 0; s < 64; ++s) *reinterpret_cast<float2*>(xbuf + xswz(pbase + 8 * s)) = b[s];
+  worker_sync(worker);
+  float2 a[16][4];
+#pragma unroll
+  for (int v = 0; v < 16; ++v)
+#pragma unroll
+    for (int r2 = 0; r2 < 2; ++r2) {
+      const float4 q = *reinterpret_cast<const float4*>(xbuf + xswz(8 * wt + 512 * v + 4 * r2));
+      a[v][2 * r2] = make_float2(q.x, q.y);
+      a[v][2 * r2 + 1] = make_float2(q.z, q.w);
+    }
+  worker_sync(worker);
+  // round B: r0, r1, r2, r9..r12
+#pragma unroll
+  for (int v = 0; v < 16; ++v) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) bf_in(a[v][i]);
+    bf2(a[v][0], a[v][1]);
+    bf2(a[v][2], a[v][3]);
+    bf2(a[v][0], a[v][2]);
+    bf2(a[v][1], a[v][3]);
+  }
+#pragma unroll
+  for (int h = 1; h < 16; h <<= 1)
+#pragma unroll
+    for (int v = 0; v < 16; ++v)
+      if ((v & h) == 0)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
+#pragma unroll
+  for (int v = 0; v < 16; ++v) IOv<D>::st8(dst, e0 + 8 * wt + 512 * v, a[v]);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Phase 2, register variant (Q <= 6): a thread owns two adjacent columns (one pair) x 2^Q rows.
+template <int Q>
+__device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
+  constexpr int R = 1 << Q;
+  const float2 sc = make_float2(scale, scale);
+  for (long long u0 = u_begin; u0 < u_end; u0 += 2 * THREADS) {
+    const long long u = u0 + 2 * threadIdx.x;  // even: the pair never straddles a plane
+    if (u >= u_end) break;
+    const long long b = u >> RB;
+    const int c = static_cast<int>(u & (ROWLEN - 1));
+    float* base = ws + (b << m) + c;
+    const float* gb = g + c;
+    float2 v[R];
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << RB)));
+    bfly_all<R>(v);
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = mul2(v[j], mul2(__ldg(reinterpret_cast<const float2*>(gb + (static_cast<long long>(j) << RB))), sc));
+    bfly_all<R>(v);
+#pragma unroll
+    for (int j = 0; j < R; ++j) __stcg(reinterpret_cast<float2*>(base + (static_cast<long long>(j) << RB)), v[j]);
+  }
+}
+
+// Phase 2, register variant for Q = 7: a thread owns one column of 128 rows as 64 pairs (j, j + 64).
+__device__ __forceinline__ void col_pass_single128(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
+  for (long long u0 = u_begin; u0 < u_end; u0 += THREADS) {
+    const long long u = u0 + threadIdx.x;
+    if (u >= u_end) break;
+    const long long b = u >> RB;
+    const int c = static_cast<int>(u & (ROWLEN - 1));
+    float* base = ws + (b << m) + c;
+    const float* gb = g + c;
+    float2 v[64];
+#pragma unroll
+    for (int j = 0; j < 64; ++j)
+      v[j] = make_float2(__ldcg(base + (static_cast<long long>(j) << RB)), __ldcg(base + (static_cast<long long>(j + 64) << RB)));
+    bfly_all<64>(v);
+#pragma unroll
+    for (int j = 0; j < 64; ++j) bf_in(v[j]);
+#pragma unroll
+    for (int j = 0; j < 64; ++j) {
+      const float2 gg = make_float2(__ldg(gb + (static_cast<long long>(j) << RB)), __ldg(gb + (static_cast<long long>(j + 64) << RB)));
+      v[j] = mul2(v[j], mul2(gg, make_float2(scale, scale)));
+    }
+#pragma unroll
+    for (int j = 0; j < 64; ++j) bf_in(v[j]);
+    bfly_all<64>(v);
+#pragma unroll
+    for (int j = 0; j < 64; ++j) {
+      __stcg(base + (static_cast<long long>(j) << RB), v[j].x);
+      __stcg(base + (static_cast<long long>(j + 64) << RB), v[j].y);
+    }
+  }
+}
+
+// The two warps (w, w + 4) that share a TMEM lane quarter meet here; TMEM stores made before the
+// barrier are visible to the other warp's loads after it.
+__device__ __forceinline__ void pair_sync(int quarter) {
+  tmem_wait_st();
+  tmem_fence_before();
+  asm volatile("bar.sync %0, %1;" ::"r"(NWORKERS + 1 + quarter), "r"(64) : "memory");
+  tmem_fence_after();
+}
+
+// Phase 2, TMEM variant (8 <= Q <= 10).  Per TMEM lane: one column half of Eh = 2^(Q - lanebit)
+// rows; the lane's 2*Et columns hold element k of warp half hw at column hw*Et + k (Et = Eh/2
+// elements per thread).  Bits: k0..k(et-1) local to a thread, k(et) = warp half (traded through
+// TMEM), and for Q = 10 the top row bit = lane bit 4 (one shuffle stage).
+//   round A: own Et elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
+//   round B: bits k6..k(et) (+ lane bit) forward, gain, back; each warp half takes k5 = hw
+//   round C: own Et elements, bits k0..k5 again, TMEM -> global
+template <int Q>
+__device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float scale, int m, long long u_begin,
+                                              long long u_end, uint32_t tlane) {
+  constexpr bool LANEBIT = Q == 10;
+  constexpr int ET_BITS = Q - 1 - (LANEBIT ? 1 : 0);  // 8, 8, 7 for Q = 10, 9, 8
+  constexpr int ET = 1 << ET_BITS;
+  constexpr int PER_PASS = LANEBIT ? 64 : 128;         // columns per pass
+  constexpr int ITA = ET / 128;                        // round A/C iterations (64 pairs each)
+  constexpr int NH = 1 << (ET_BITS - 5);               // high combinations in round B (incl. warp half)
+  constexpr int W = 64 / NH;                           // pairs per high combination
+  constexpr int ITB = 16 / W;                          // round B iterations
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int quarter = warp & 3, hw = warp >> 2;
+  const int slot = LANEBIT ? quarter * 16 + (lane & 15) : quarter * 32 + lane;
+  const int h = LANEBIT ? (lane >> 4) : 0;
+  const float2 sgn = h ? make_float2(-1.f, -1.f) : make_float2(1.f, 1.f);
+  const float2 sc = make_float2(scale, scale);
+  for (long long u0 = u_begin; u0 < u_end; u0 += PER_PASS) {
+    const long long u = u0 + slot;
+    const bool active = u < u_end;
+    const long long uu = active ? u : u_begin;  // inactive lanes compute on a valid column, never store
+    const long long b = uu >> RB;
+    const int c = static_cast<int>(uu & (ROWLEN - 1));
+    float* colp = ws + (b << m) + c + (static_cast<long long>(h) << (9 + RB));
+    const float* gcol = g + c + (static_cast<long long>(h) << (9 + RB));
+    float* own = colp + (static_cast<long long>(hw * ET) << RB);
+    // round A
+#pragma unroll 1
+    for (int it = 0; it < ITA; ++it) {
+      float2 v[64];
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
+        v[k] = make_float2(__ldcg(own + (k0 << RB)), __ldcg(own + (k1 << RB)));
+      }
+      bfly_all<64>(v);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float lo[16], hi[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          lo[i] = v[16 * q + i].x;
+          hi[i] = v[16 * q + i].y;
+        }
+        tmem_st16(tlane + hw * ET + 64 * it + 16 * q, lo);
+        tmem_st16(tlane + hw * ET + ET / 2 + 64 * it + 16 * q, hi);
+      }
+    }
+    pair_sync(quarter);
+    // round B
+#pragma unroll 1
+    for (int it = 0; it < ITB; ++it) {
+      float2 v[NH][W];
+#pragma unroll
+      for (int s = 0; s < NH; ++s) {
+        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+        const uint32_t col = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+        for (int q = 0; q < 2 * W / 16; ++q) {
+          float t[16];
+          tmem_ld16(tlane + col + 16 * q, t);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[s][8 * q + i] = make_float2(t[2 * i], t[2 * i + 1]);
+        }
+      }
+      tmem_wait_ld();
+#pragma unroll
+      for (int hh = 1; hh < NH; hh <<= 1)
+#pragma unroll
+        for (int s = 0; s < NH; ++s)
+          if ((s & hh) == 0)
+#pragma unroll
+            for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
+      if (LANEBIT) {
+#pragma unroll
+        for (int s = 0; s < NH; ++s)
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            const float2 p = make_float2(__shfl_xor_sync(0xffffffffu, v[s][w].x, 16), __shfl_xor_sync(0xffffffffu, v[s][w].y, 16));
+            v[s][w] = fma2(v[s][w], sgn, p);
+          }
+      }
+#pragma unroll
+      for (int s = 0; s < NH; ++s) {
+        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+          const long long j = j0 + 2 * w;
+          const float2 gg = make_float2(__ldg(gcol + (j << RB)), __ldg(gcol + ((j + 1) << RB)));
+          v[s][w] = mul2(v[s][w], mul2(gg, sc));
+        }
+      }
+      if (LANEBIT) {
+#pragma unroll
+        for (int s = 0; s < NH; ++s)
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            const float2 p = make_float2(__shfl_xor_sync(0xffffffffu, v[s][w].x, 16), __shfl_xor_sync(0xffffffffu, v[s][w].y, 16));
+            v[s][w] = fma2(v[s][w], sgn, p);
+          }
+      }
+#pragma unroll
+      for (int hh = 1; hh < NH; hh <<= 1)
+#pragma unroll
+        for (int s = 0; s < NH; ++s)
+          if ((s & hh) == 0)
+#pragma unroll
+            for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
+#pragma unroll
+      for (int s = 0; s < NH; ++s) {
+        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+        const uint32_t col = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+        for (int q = 0; q < 2 * W / 16; ++q) {
+          float t[16];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            t[2 * i] = v[s][8 * q + i].x;
+            t[2 * i + 1] = v[s][8 * q + i].y;
+          }
+          tmem_st16(tlane + col + 16 * q, t);
+        }
+      }
+    }
+    pair_sync(quarter);
+    // round C
+#pragma unroll 1
+    for (int it = 0; it < ITA; ++it) {
+      float2 v[64];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float lo[16], hi[16];
+        tmem_ld16(tlane + hw * ET + 64 * it + 16 * q, lo);
+        tmem_ld16(tlane + hw * ET + ET / 2 + 64 * it + 16 * q, hi);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[16 * q + i] = make_float2(lo[i], hi[i]);
+      }
+      tmem_wait_ld();
+      bfly_all<64>(v);
+      if (active) {
+#pragma unroll
+        for (int k = 0; k < 64; ++k) {
+          const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
+          __stcg(own + (k0 << RB), v[k].x);
+          __stcg(own + (k1 << RB), v[k].y);
+        }
+      }
+    }
+    // the next pass's round A overwrites only this thread's own columns, which the other warp
+    // of the pair stopped reading at the second pair_sync
+  }
+}
+
+// L2 prefetch of the first G_PREFETCH_EIGHTHS/8 of G's rows for this CTA's phase-2 columns.
+__device__ __forceinline__ void prefetch_gain_rows(const float* g, int q, long long cb, long long ce) {
+  if (ce <= cb) return;
+  const long long c_lo = cb & (ROWLEN - 1);
+  const long long c_hi = min(static_cast<long long>(ROWLEN), c_lo + (ce - cb));
+  const uint32_t bytes = static_cast<uint32_t>((c_hi - c_lo) * 4);  // multiple of 32
+  const int rows = ((1 << q) * G_PREFETCH_EIGHTHS) / 8;
+  for (int j = threadIdx.x; j < rows; j += THREADS) {
+    const float* p = g + (static_cast<long long>(j) << RB) + c_lo;
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Forward kernel: persistent cooperative grid (one CTA per SM), plane groups of P.gp planes,
+// three phases.  Q = m - 13 is a template parameter so that every register array has a static size.
+template <int D, int Q>
+__global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ int flag;
+  __shared__ uint32_t tmem_slot;
+  constexpr bool USE_TMEM = Q >= 8;
+  float* xbuf_all = reinterpret_cast<float*>(smem_raw);
+  const int worker = threadIdx.x / WORKER, wt = threadIdx.x % WORKER;
+  float* xbuf = xbuf_all + worker * ROWLEN;
+  float* ws = static_cast<float*>(P.ws);
+  const float* g = static_cast<const float*>(P.g);
+  const int m = RB + Q;
+  uint32_t tlane = 0;
+  if constexpr (USE_TMEM) {
+    if (threadIdx.x < 32) tmem_alloc_512(&tmem_slot);
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    tlane = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16);
+  }
+  for (long long b0 = 0; b0 < P.B; b0 += P.gp) {
+    const long long nb = min(static_cast<long long>(P.gp), P.B - b0);
+    const long long rows = nb << Q;
+    const long long rb = rows * blockIdx.x / gridDim.x, re = rows * (blockIdx.x + 1) / gridDim.x;
+    // phase-2 column range: balanced, aligned to 8 columns
+    const long long cols = nb << RB;
+    const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
+    const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
+    // phase 1: X -> ws, row bits
+    if constexpr (USE_TMEM) prefetch_gain_rows(g, Q, cb, ce);
+    for (long long r = rb + worker; r < re; r += NWORKERS)
+      row_forward_in<D>(P.x, ((b0 << m) + (r << RB)), ws + (r << RB), xbuf, wt, worker);
+    if (!grid_sync(P.bar, &flag)) break;
+    // phase 2: column bits, gain, column bits
+    if constexpr (USE_TMEM) col_pass_tmem<Q>(ws, g, P.scale, m, cb, ce, tlane);
+    else if constexpr (Q == 7) col_pass_single128(ws, g, P.scale, m, cb, ce);
+    else col_pass_pairs<Q>(ws, g, P.scale, m, cb, ce);
+    if (!grid_sync(P.bar, &flag)) break;
+    // phase 3: ws -> Y, row bits
+    for (long long r = rb + worker; r < re; r += NWORKERS)
+      row_forward_out<D>(ws + (r << RB), P.y, ((b0 << m) + (r << RB)), xbuf, wt, worker);
+    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) break;
+  }
+  if constexpr (USE_TMEM) {
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    if (threadIdx.x < 32) tmem_dealloc_512(tmem_slot);
+  }
+}
+
+}  // namespace fast
+}  // namespace whtmix

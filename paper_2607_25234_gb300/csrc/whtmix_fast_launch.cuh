@@ -1,0 +1,77 @@
+// whtmix_fast_launch.cuh -- host-side launcher of the fast forward kernels for one I/O dtype.
+// Included by whtmix_fast_f32.cu and whtmix_fast_bf16.cu (one translation unit each, compiled in
+// parallel).  Returns a cudaError_t; the C ABI maps it to a status.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <map>
+#include <mutex>
+
+#include "whtmix_fast.cuh"
+
+namespace whtmix {
+namespace fast {
+
+// Resident CTAs per SM for one kernel and smem size, per device (first query also raises the
+// kernel's dynamic shared memory limit).
+inline cudaError_t occupancy_cached(const void* kernel, size_t smem, int* occ) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, int> cache;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = cache.find({dev, kernel});
+  if (it != cache.end()) {
+    *occ = it->second;
+    return cudaSuccess;
+  }
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(occ, kernel, THREADS, smem);
+  if (e != cudaSuccess) return e;
+  if (*occ < 1) return cudaErrorInvalidConfiguration;
+  cache[{dev, kernel}] = *occ;
+  return cudaSuccess;
+}
+
+// Every variant requests more than half an SM's shared memory, so exactly one CTA runs per SM:
+// two CTAs on one SM would both ask for all 512 TMEM columns, and the second would wait in
+// tcgen05.alloc while the first waits for it at the device-wide barrier.
+template <int D, int Q>
+cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
+  const size_t smem = SMEM_BYTES;
+  const void* k = reinterpret_cast<const void*>(k_forward_fast<D, Q>);
+  int occ = 0;
+  cudaError_t e = occupancy_cached(k, smem, &occ);
+  if (e != cudaSuccess) return e;
+  if (occ != 1) return cudaErrorInvalidConfiguration;
+  Params p = P;
+  void* args[] = {&p};
+  return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, smem, stream);
+}
+
+template <int D>
+cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
+  switch (P.m - RB) {
+    case 1: return launch_one<D, 1>(P, sms, stream);
+    case 2: return launch_one<D, 2>(P, sms, stream);
+    case 3: return launch_one<D, 3>(P, sms, stream);
+    case 4: return launch_one<D, 4>(P, sms, stream);
+    case 5: return launch_one<D, 5>(P, sms, stream);
+    case 6: return launch_one<D, 6>(P, sms, stream);
+    case 7: return launch_one<D, 7>(P, sms, stream);
+    case 8: return launch_one<D, 8>(P, sms, stream);
+    case 9: return launch_one<D, 9>(P, sms, stream);
+    case 10: return launch_one<D, 10>(P, sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// Entry points defined in whtmix_fast_f32.cu / whtmix_fast_bf16.cu.
+cudaError_t forward_f32(const Params& P, int sms, cudaStream_t stream);
+cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream);
+
+}  // namespace fast
+}  // namespace whtmix

@@ -287,10 +287,11 @@ __device__ __forceinline__ bool grid_sync(GridBarrier* bar, int* flag) {
       __threadfence();
       atomicAdd(&bar->gen, 1u);
     } else {
+      // Spin on the generation word (no sleep: the wait is ~1 us and a sleep quantum would add
+      // to it); the clock is read once per 256 polls to bound the wait.
       const unsigned long long t0 = global_ns();
-      while (ld_acquire(&bar->gen) == gen) {
-        __nanosleep(64);
-        if (global_ns() - t0 > BARRIER_TIMEOUT_NS) {
+      for (unsigned int polls = 1; ld_acquire(&bar->gen) == gen; ++polls) {
+        if ((polls & 255u) == 0 && global_ns() - t0 > BARRIER_TIMEOUT_NS) {
           atomicOr(&bar->err, 1u);
           ok = 0;
           break;

@@ -124,7 +124,10 @@ def test_train_16x8192x256_bf16_forward_backward():
 
 SWEEP = [(1, 1, 1), (3, 1, 1), (5, 1, 8), (7, 8, 1), (3, 2, 2), (9, 4, 16), (2, 16, 4), (33, 32, 8),
          (3, 64, 128), (2, 128, 64), (1, 8192, 1), (1, 1, 8192), (2, 1, 16384), (3, 16384, 1),
-         (2, 64, 256), (3, 512, 32), (1, 2048, 64), (2, 256, 1024), (1, 1 << 18, 2), (1, 2, 1 << 18)]
+         (2, 64, 256), (3, 512, 32), (1, 2048, 64), (2, 256, 1024), (1, 1 << 18, 2), (1, 2, 1 << 18),
+         # every column height of the fast forward: N*C = 2^(13+Q), Q = 1..10
+         (2, 128, 256), (3, 2048, 8), (2, 1024, 1024), (3, 256, 4096), (1, 4096, 1024), (2, 8192, 512),
+         (1, 1 << 20, 8), (1, 16, 1 << 19)]
 
 
 @pytest.mark.parametrize("B,N,C", SWEEP)
