@@ -13,8 +13,8 @@
 //     elements; otherwise the two warps (w, w+4) that share a TMEM lane quarter hold one column
 //     per lane (Blackwell tensor memory as per-thread storage, 256 fp32 per thread), trade the
 //     bit between their halves through TMEM, and a 1024-element column adds one shuffle stage;
-//   * column ranges are balanced and aligned to 8 columns (32-byte sectors); G is prefetched into
-//     L2 during phase 1, which is bound by its writes and leaves HBM reads idle.
+//   * column ranges are balanced and aligned to 8 columns (32-byte sectors); for 1024-row columns
+//     the gains are staged through shared memory with cp.async one round-B iteration ahead.
 // Phase 2's flat-index bits are the row bits [13, m); the gain multiplies by G[j*2^13 + c]/L.
 #pragma once
 
@@ -30,7 +30,11 @@ constexpr int WORKER = 64;     // threads per row worker
 constexpr int NWORKERS = THREADS / WORKER;
 // four row exchange buffers (128 KiB): more than half an SM, so exactly one CTA runs per SM
 constexpr size_t SMEM_BYTES = NWORKERS * ROWLEN * sizeof(float);
-constexpr int G_PREFETCH_EIGHTHS = 8;  // share of G's rows (in eighths) prefetched into L2 in phase 1
+static_assert(SMEM_BYTES >= 128 * THREADS * sizeof(float), "phase 2 stages 128 gains per thread in the row buffers");
+#ifndef G_PREFETCH_EIGHTHS_DEFAULT
+#define G_PREFETCH_EIGHTHS_DEFAULT 0
+#endif
+constexpr int G_PREFETCH_EIGHTHS = G_PREFETCH_EIGHTHS_DEFAULT;  // share of G's rows (in eighths) prefetched into L2 in phase 1
 
 // ---------------------------------------------------------------------------------------------
 // packed fp32 pairs
@@ -316,6 +320,14 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
   }
 }
 
+// Asynchronous 4-byte global -> shared copies (no registers held while in flight).
+__device__ __forceinline__ void cp_async4(float* smem_dst, const float* gsrc) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // The two warps (w, w + 4) that share a TMEM lane quarter meet here; TMEM stores made before the
 // barrier are visible to the other warp's loads after it.
 __device__ __forceinline__ void pair_sync(int quarter) {
@@ -332,9 +344,12 @@ __device__ __forceinline__ void pair_sync(int quarter) {
 //   round A: own Et elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
 //   round B: bits k6..k(et) (+ lane bit) forward, gain, back; each warp half takes k5 = hw
 //   round C: own Et elements, bits k0..k5 again, TMEM -> global
+//   G for round B is staged in shared memory (gstage, the idle row buffers) with cp.async, one
+//   round-B iteration ahead: value v of thread t sits at gstage[v * THREADS + t], and every thread
+//   reads back only what it copied itself, so no barrier is needed.
 template <int Q>
 __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float scale, int m, long long u_begin,
-                                              long long u_end, uint32_t tlane) {
+                                              long long u_end, uint32_t tlane, float* gstage) {
   constexpr bool LANEBIT = Q == 10;
   constexpr int ET_BITS = Q - 1 - (LANEBIT ? 1 : 0);  // 8, 8, 7 for Q = 10, 9, 8
   constexpr int ET = 1 << ET_BITS;
@@ -343,6 +358,9 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
   constexpr int NH = 1 << (ET_BITS - 5);               // high combinations in round B (incl. warp half)
   constexpr int W = 64 / NH;                           // pairs per high combination
   constexpr int ITB = 16 / W;                          // round B iterations
+  // With the shuffle stages in round B there are no spare registers to hoist the G loads above
+  // them, so for Q = 10 G is staged ahead through shared memory; otherwise it is loaded directly.
+  constexpr bool STAGE_G = LANEBIT;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int quarter = warp & 3, hw = warp >> 2;
   const int slot = LANEBIT ? quarter * 16 + (lane & 15) : quarter * 32 + lane;
@@ -358,6 +376,22 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
     float* colp = ws + (b << m) + c + (static_cast<long long>(h) << (9 + RB));
     const float* gcol = g + c + (static_cast<long long>(h) << (9 + RB));
     float* own = colp + (static_cast<long long>(hw * ET) << RB);
+    // G rows of round-B iteration `it`, in the order the gain step consumes them
+    auto stage_gain = [&](int it) {
+#pragma unroll
+      for (int s = 0; s < NH; ++s) {
+        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+          const int vi = 2 * (s * W + w);
+          cp_async4(gstage + vi * THREADS + threadIdx.x, gcol + ((j0 + 2 * w) << RB));
+          cp_async4(gstage + (vi + 1) * THREADS + threadIdx.x, gcol + ((j0 + 2 * w + 1) << RB));
+        }
+      }
+      cp_async_commit();
+    };
+    if constexpr (STAGE_G) stage_gain(0);
     // round A
 #pragma unroll 1
     for (int it = 0; it < ITA; ++it) {
@@ -414,15 +448,28 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
             v[s][w] = fma2(v[s][w], sgn, p);
           }
       }
+      if constexpr (STAGE_G) {
+        cp_async_wait_all();
 #pragma unroll
-      for (int s = 0; s < NH; ++s) {
-        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+        for (int s = 0; s < NH; ++s)
 #pragma unroll
-        for (int w = 0; w < W; ++w) {
-          const long long j = j0 + 2 * w;
-          const float2 gg = make_float2(__ldg(gcol + (j << RB)), __ldg(gcol + ((j + 1) << RB)));
-          v[s][w] = mul2(v[s][w], mul2(gg, sc));
+          for (int w = 0; w < W; ++w) {
+            const int vi = 2 * (s * W + w);
+            const float2 gg = make_float2(gstage[vi * THREADS + threadIdx.x], gstage[(vi + 1) * THREADS + threadIdx.x]);
+            v[s][w] = mul2(v[s][w], mul2(gg, sc));
+          }
+        if (it + 1 < ITB) stage_gain(it + 1);
+      } else {
+#pragma unroll
+        for (int s = 0; s < NH; ++s) {
+          const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+          const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            const long long j = j0 + 2 * w;
+            const float2 gg = make_float2(__ldg(gcol + (j << RB)), __ldg(gcol + ((j + 1) << RB)));
+            v[s][w] = mul2(v[s][w], mul2(gg, sc));
+          }
         }
       }
       if (LANEBIT) {
@@ -531,12 +578,12 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
     const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
     // phase 1: X -> ws, row bits
-    if constexpr (USE_TMEM) prefetch_gain_rows(g, Q, cb, ce);
+    if constexpr (USE_TMEM && G_PREFETCH_EIGHTHS > 0) prefetch_gain_rows(g, Q, cb, ce);
     for (long long r = rb + worker; r < re; r += NWORKERS)
       row_forward_in<D>(P.x, ((b0 << m) + (r << RB)), ws + (r << RB), xbuf, wt, worker);
     if (!grid_sync(P.bar, &flag)) break;
     // phase 2: column bits, gain, column bits
-    if constexpr (USE_TMEM) col_pass_tmem<Q>(ws, g, P.scale, m, cb, ce, tlane);
+    if constexpr (USE_TMEM) col_pass_tmem<Q>(ws, g, P.scale, m, cb, ce, tlane, xbuf_all);
     else if constexpr (Q == 7) col_pass_single128(ws, g, P.scale, m, cb, ce);
     else col_pass_pairs<Q>(ws, g, P.scale, m, cb, ce);
     if (!grid_sync(P.bar, &flag)) break;
