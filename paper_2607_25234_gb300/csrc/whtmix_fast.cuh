@@ -8,7 +8,9 @@
 //   * butterflies run on register pairs with packed add/sub.f32x2 (half the instructions);
 //   * one CTA of 8 warps per SM; phase 1 / phase 3 work on rows of 2^13 elements, one row per
 //     64-thread worker (4 per CTA), 128 elements per thread, exactly one shared-memory exchange
-//     per row (conflict-free XOR swizzle), on a balanced contiguous range of rows per SM;
+//     per row (conflict-free XOR swizzle), on a balanced contiguous range of rows per SM; each
+//     worker's next row is prefetched with cp.async while the current one is processed, and the
+//     workspace stores rows bit-permuted so that every row access is a contiguous 256-byte span;
 //   * phase 2 gives columns to threads: whole columns in registers when a column has <= 128
 //     elements; otherwise the two warps (w, w+4) that share a TMEM lane quarter hold one column
 //     per lane (Blackwell tensor memory as per-thread storage, 256 fp32 per thread), trade the
@@ -28,13 +30,13 @@ constexpr int RB = 13;         // row bits
 constexpr int ROWLEN = 1 << RB;
 constexpr int WORKER = 64;     // threads per row worker
 constexpr int NWORKERS = THREADS / WORKER;
-// four row exchange buffers (128 KiB): more than half an SM, so exactly one CTA runs per SM
-constexpr size_t SMEM_BYTES = NWORKERS * ROWLEN * sizeof(float);
-static_assert(SMEM_BYTES >= 128 * THREADS * sizeof(float), "phase 2 stages 128 gains per thread in the row buffers");
-#ifndef G_PREFETCH_EIGHTHS_DEFAULT
-#define G_PREFETCH_EIGHTHS_DEFAULT 0
-#endif
-constexpr int G_PREFETCH_EIGHTHS = G_PREFETCH_EIGHTHS_DEFAULT;  // share of G's rows (in eighths) prefetched into L2 in phase 1
+// shared memory: four row exchange buffers (128 KiB) and four 16 KiB row staging areas for
+// cp.async prefetch of each worker's next row.  More than half an SM, so exactly one CTA per SM.
+constexpr int STAGE_FLOATS = 4096;
+constexpr size_t SMEM_XBUF_BYTES = NWORKERS * ROWLEN * sizeof(float);
+constexpr size_t SMEM_BYTES = SMEM_XBUF_BYTES + NWORKERS * STAGE_FLOATS * sizeof(float);
+static_assert(SMEM_XBUF_BYTES >= 128 * THREADS * sizeof(float), "phase 2 stages 128 gains per thread in the row buffers");
+static_assert(SMEM_BYTES <= 227 * 1024, "shared memory per CTA");
 
 // ---------------------------------------------------------------------------------------------
 // packed fp32 pairs
@@ -133,6 +135,18 @@ __device__ __forceinline__ int xswz(int r) {
   return r ^ (((r >> 5) & 1) << 2) ^ (((r >> 9) & 1) << 3) ^ (((r >> 10) & 1) << 4);
 }
 
+// Workspace rows are stored with their 13 index bits permuted (sigma), so that layout P's lanes
+// (r1, r2, r9, r10, r11, plus the in-register pair bit r0) cover 64 consecutive floats: phase 1's
+// stores and phase 3's loads are one 256-byte span per warp instruction.  Storage position s of
+// row element r: s = (r0, r1, r2, r9, r10, r11, r3, r4, r5, r6, r7, r8, r12) from bit 0 up.
+// Phase 2 works in storage positions and maps back to the logical column only to index G.
+__device__ __forceinline__ int sigma(int r) {
+  return (r & 7) | (((r >> 9) & 7) << 3) | (((r >> 3) & 63) << 6) | (r & 4096);
+}
+__device__ __forceinline__ int sigma_inv(int s) {
+  return (s & 7) | (((s >> 6) & 63) << 3) | (((s >> 3) & 7) << 9) | (s & 4096);
+}
+
 __device__ __forceinline__ void worker_sync(int worker) {
   asm volatile("bar.sync %0, %1;" ::"r"(worker + 1), "r"(WORKER) : "memory");
 }
@@ -174,16 +188,86 @@ template <> struct IOv<DT_F32> {
 };
 
 // ---------------------------------------------------------------------------------------------
+// Asynchronous global -> shared copies (no registers held while in flight).
+__device__ __forceinline__ void cp_async16(float* smem_dst, const void* gsrc) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async8(float* smem_dst, const void* gsrc) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(s), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async4(float* smem_dst, const float* gsrc) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// Row prefetch.  Every thread copies exactly the 16-byte (8-byte) chunks it will read back
+// itself, so the staging area needs no barrier; chunk k of thread wt sits at (k * 64 + wt), which
+// makes each warp's read-back one contiguous 512-byte (256-byte) span.
+// Phase 1 stages a whole bf16 row (16 vectors of 8 elements) or the first half of an fp32 row.
+template <int D>
+__device__ __forceinline__ void stage_row_in(const void* src, long long e0, float* stg, int wt) {
+  if constexpr (D == DT_BF16) {
+#pragma unroll
+    for (int v = 0; v < 16; ++v)
+      cp_async16(stg + (v * 64 + wt) * 4, static_cast<const unsigned short*>(src) + e0 + 8 * wt + 512 * v);
+  } else {
+#pragma unroll
+    for (int v = 0; v < 8; ++v)
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2)
+        cp_async16(stg + ((2 * v + h2) * 64 + wt) * 4, static_cast<const float*>(src) + e0 + 8 * wt + 512 * v + 4 * h2);
+  }
+  cp_async_commit();
+}
+// Phase 3 stages the first 32 of the 64 pairs each thread reads in layout P.
+__device__ __forceinline__ int pbase_of(int wt) { return 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2); }
+__device__ __forceinline__ void stage_row_out(const float* src_ws, float* stg, int wt) {
+  const int pbase = pbase_of(wt);
+#pragma unroll
+  for (int s = 0; s < 32; ++s) cp_async8(stg + (s * 64 + wt) * 2, src_ws + sigma(pbase + 8 * s));
+  cp_async_commit();
+}
+
+// ---------------------------------------------------------------------------------------------
 // Phase 1 row: X (dtype D) -> workspace (fp32), butterflies on all 13 row bits.
 //   layout V: thread wt holds r0..r2 (8-vectors) x r9..r12 (16 vectors); wt = r3..r8.
 //     round A: bits r1, r2, r9..r12 (pairs on r0).
 //   exchange through smem, then layout P: thread holds pairs (r0) x r3..r8; wt bits =
 //     (r1, r2, r9, r10, r11, r12).  round B: r0 (inside the pairs) and r3..r8.
+// The row arrives through the staging area (prefetched while the previous row was processed);
+// the next row's prefetch (e0_next >= 0) is issued as soon as this row is in registers.
 template <int D>
-__device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, int wt, int worker) {
+__device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, float* stg,
+                                               int wt, int worker, long long e0_next) {
   float2 a[16][4];  // [v = r9..r12][r1 + 2 r2]
+  if constexpr (D == DT_F32) {
 #pragma unroll
-  for (int v = 0; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + 512 * v, a[v]);
+    for (int v = 8; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + 512 * v, a[v]);
+  }
+  cp_async_wait_all();
+  if constexpr (D == DT_BF16) {
+#pragma unroll
+    for (int v = 0; v < 16; ++v) {
+      const uint4 u = *reinterpret_cast<const uint4*>(stg + (v * 64 + wt) * 4);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[v][i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+    }
+  } else {
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const float4 q0 = *reinterpret_cast<const float4*>(stg + ((2 * v) * 64 + wt) * 4);
+      const float4 q1 = *reinterpret_cast<const float4*>(stg + ((2 * v + 1) * 64 + wt) * 4);
+      a[v][0] = make_float2(q0.x, q0.y);
+      a[v][1] = make_float2(q0.z, q0.w);
+      a[v][2] = make_float2(q1.x, q1.y);
+      a[v][3] = make_float2(q1.z, q1.w);
+    }
+  }
   // round A
 #pragma unroll
   for (int v = 0; v < 16; ++v) {
@@ -199,6 +283,7 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
       if ((v & h) == 0)
 #pragma unroll
         for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
+  if (e0_next >= 0) stage_row_in<D>(src, e0_next, stg, wt);
   // exchange V -> P
 #pragma unroll
   for (int v = 0; v < 16; ++v)
@@ -208,7 +293,7 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
       *reinterpret_cast<float4*>(xbuf + xswz(r)) = make_float4(a[v][2 * r2].x, a[v][2 * r2].y, a[v][2 * r2 + 1].x, a[v][2 * r2 + 1].y);
     }
   worker_sync(worker);
-  const int pbase = 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2);  // r1, r2, r9..r12
+  const int pbase = pbase_of(wt);  // r1, r2, r9..r12
   float2 b[64];  // [s = r3..r8]
 #pragma unroll
   for (int s = 0; s < 64; ++s) b[s] = *reinterpret_cast<const float2*>(xbuf + xswz(pbase + 8 * s));
@@ -218,17 +303,24 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
   for (int s = 0; s < 64; ++s) bf_in(b[s]);
   bfly_all<64>(b);
 #pragma unroll
-  for (int s = 0; s < 64; ++s) __stcg(reinterpret_cast<float2*>(dst_ws + pbase + 8 * s), b[s]);
+  for (int s = 0; s < 64; ++s) __stcg(reinterpret_cast<float2*>(dst_ws + sigma(pbase + 8 * s)), b[s]);
 }
 
 // Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all 13 row bits (mirror of phase 1).
+// The first half of the row's pairs arrives through the staging area; src_next (if not null) is
+// the next row, whose prefetch is issued once this row is in registers.
 template <int D>
-__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, float* xbuf, int wt, int worker) {
-  const int pbase = 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2);
+__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, float* xbuf, float* stg,
+                                                int wt, int worker, const float* src_next) {
+  const int pbase = pbase_of(wt);
   float2 b[64];
 #pragma unroll
-  for (int s = 0; s < 64; ++s) b[s] = __ldcg(reinterpret_cast<const float2*>(src_ws + pbase + 8 * s));
+  for (int s = 32; s < 64; ++s) b[s] = __ldcg(reinterpret_cast<const float2*>(src_ws + sigma(pbase + 8 * s)));
+  cp_async_wait_all();
+#pragma unroll
+  for (int s = 0; s < 32; ++s) b[s] = *reinterpret_cast<const float2*>(stg + (s * 64 + wt) * 2);
   bfly_all<64>(b);  // round A: r3..r8
+  if (src_next != nullptr) stage_row_out(src_next, stg, wt);
 #pragma unroll
   for (int s = 0; s < 64; ++s) *reinterpret_cast<float2*>(xbuf + xswz(pbase + 8 * s)) = b[s];
   worker_sync(worker);
@@ -273,9 +365,9 @@ __device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float 
     const long long u = u0 + 2 * threadIdx.x;  // even: the pair never straddles a plane
     if (u >= u_end) break;
     const long long b = u >> RB;
-    const int c = static_cast<int>(u & (ROWLEN - 1));
-    float* base = ws + (b << m) + c;
-    const float* gb = g + c;
+    const int sp = static_cast<int>(u & (ROWLEN - 1));  // storage position (even); sp + 1 is column c + 1
+    float* base = ws + (b << m) + sp;
+    const float* gb = g + sigma_inv(sp);
     float2 v[R];
 #pragma unroll
     for (int j = 0; j < R; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << RB)));
@@ -294,9 +386,9 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
     const long long u = u0 + threadIdx.x;
     if (u >= u_end) break;
     const long long b = u >> RB;
-    const int c = static_cast<int>(u & (ROWLEN - 1));
-    float* base = ws + (b << m) + c;
-    const float* gb = g + c;
+    const int sp = static_cast<int>(u & (ROWLEN - 1));
+    float* base = ws + (b << m) + sp;
+    const float* gb = g + sigma_inv(sp);
     float2 v[64];
 #pragma unroll
     for (int j = 0; j < 64; ++j)
@@ -319,14 +411,6 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
     }
   }
 }
-
-// Asynchronous 4-byte global -> shared copies (no registers held while in flight).
-__device__ __forceinline__ void cp_async4(float* smem_dst, const float* gsrc) {
-  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gsrc) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // The two warps (w, w + 4) that share a TMEM lane quarter meet here; TMEM stores made before the
 // barrier are visible to the other warp's loads after it.
@@ -372,9 +456,9 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
     const bool active = u < u_end;
     const long long uu = active ? u : u_begin;  // inactive lanes compute on a valid column, never store
     const long long b = uu >> RB;
-    const int c = static_cast<int>(uu & (ROWLEN - 1));
-    float* colp = ws + (b << m) + c + (static_cast<long long>(h) << (9 + RB));
-    const float* gcol = g + c + (static_cast<long long>(h) << (9 + RB));
+    const int sp = static_cast<int>(uu & (ROWLEN - 1));  // storage position of the column
+    float* colp = ws + (b << m) + sp + (static_cast<long long>(h) << (9 + RB));
+    const float* gcol = g + sigma_inv(sp) + (static_cast<long long>(h) << (9 + RB));
     float* own = colp + (static_cast<long long>(hw * ET) << RB);
     // G rows of round-B iteration `it`, in the order the gain step consumes them
     auto stage_gain = [&](int it) {
@@ -533,19 +617,6 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
   }
 }
 
-// L2 prefetch of the first G_PREFETCH_EIGHTHS/8 of G's rows for this CTA's phase-2 columns.
-__device__ __forceinline__ void prefetch_gain_rows(const float* g, int q, long long cb, long long ce) {
-  if (ce <= cb) return;
-  const long long c_lo = cb & (ROWLEN - 1);
-  const long long c_hi = min(static_cast<long long>(ROWLEN), c_lo + (ce - cb));
-  const uint32_t bytes = static_cast<uint32_t>((c_hi - c_lo) * 4);  // multiple of 32
-  const int rows = ((1 << q) * G_PREFETCH_EIGHTHS) / 8;
-  for (int j = threadIdx.x; j < rows; j += THREADS) {
-    const float* p = g + (static_cast<long long>(j) << RB) + c_lo;
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-  }
-}
-
 // ---------------------------------------------------------------------------------------------
 // Forward kernel: persistent cooperative grid (one CTA per SM), plane groups of P.gp planes,
 // three phases.  Q = m - 13 is a template parameter so that every register array has a static size.
@@ -558,6 +629,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   float* xbuf_all = reinterpret_cast<float*>(smem_raw);
   const int worker = threadIdx.x / WORKER, wt = threadIdx.x % WORKER;
   float* xbuf = xbuf_all + worker * ROWLEN;
+  float* stg = xbuf_all + NWORKERS * ROWLEN + worker * STAGE_FLOATS;
   float* ws = static_cast<float*>(P.ws);
   const float* g = static_cast<const float*>(P.g);
   const int m = RB + Q;
@@ -578,9 +650,12 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
     const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
     // phase 1: X -> ws, row bits
-    if constexpr (USE_TMEM && G_PREFETCH_EIGHTHS > 0) prefetch_gain_rows(g, Q, cb, ce);
-    for (long long r = rb + worker; r < re; r += NWORKERS)
-      row_forward_in<D>(P.x, ((b0 << m) + (r << RB)), ws + (r << RB), xbuf, wt, worker);
+    if (rb + worker < re) stage_row_in<D>(P.x, (b0 << m) + ((rb + worker) << RB), stg, wt);
+    for (long long r = rb + worker; r < re; r += NWORKERS) {
+      const long long rn = r + NWORKERS;
+      row_forward_in<D>(P.x, (b0 << m) + (r << RB), ws + (r << RB), xbuf, stg, wt, worker,
+                        rn < re ? (b0 << m) + (rn << RB) : -1);
+    }
     if (!grid_sync(P.bar, &flag)) break;
     // phase 2: column bits, gain, column bits
     if constexpr (USE_TMEM) col_pass_tmem<Q>(ws, g, P.scale, m, cb, ce, tlane, xbuf_all);
@@ -588,8 +663,12 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     else col_pass_pairs<Q>(ws, g, P.scale, m, cb, ce);
     if (!grid_sync(P.bar, &flag)) break;
     // phase 3: ws -> Y, row bits
-    for (long long r = rb + worker; r < re; r += NWORKERS)
-      row_forward_out<D>(ws + (r << RB), P.y, ((b0 << m) + (r << RB)), xbuf, wt, worker);
+    if (rb + worker < re) stage_row_out(ws + ((rb + worker) << RB), stg, wt);
+    for (long long r = rb + worker; r < re; r += NWORKERS) {
+      const long long rn = r + NWORKERS;
+      row_forward_out<D>(ws + (r << RB), P.y, (b0 << m) + (r << RB), xbuf, stg, wt, worker,
+                         rn < re ? ws + (rn << RB) : nullptr);
+    }
     if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) break;
   }
   if constexpr (USE_TMEM) {
