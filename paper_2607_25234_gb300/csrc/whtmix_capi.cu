@@ -185,7 +185,7 @@ int launch(K kernel, bool cooperative, int sms, long long max_units, size_t smem
 
 // The fast forward (whtmix_fast.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^23.
 bool use_fast_forward(int dtype, int m) {
-  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m > fast::RB && m <= fast::RB + 10;
+  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 23;
 }
 
 template <int D>

@@ -4,20 +4,24 @@
 // Same three phases as the generic plan M (Section III-B map; see whtmix_kernels.cuh), written
 // for the instruction and latency budget of the path: the butterflies need 2 log2(NC) fp32 adds
 // per element, which at N*C = 2^23 on 152 SMs is about as long as streaming X, G and Y through
-// HBM, and every SM must keep ~100 KB of loads in flight to hide memory latency.  So:
+// HBM.  A plane of 2^m elements is viewed as 2^Q rows of 2^R contiguous elements (R = 13, or 14
+// for m >= 22, so that Q <= 9):
+//   phase 1  every row: its R bits forward                              X  -> workspace
+//   phase 2  every column: its Q bits forward, gain G/L, Q bits again   workspace -> workspace
+//   phase 3  every row: its R bits again                                workspace -> Y
+// with a bounded device-wide barrier between phases.  Design points:
 //   * butterflies run on register pairs with packed add/sub.f32x2 (half the instructions);
-//   * one CTA of 8 warps per SM; phase 1 / phase 3 work on rows of 2^13 elements, one row per
-//     64-thread worker (4 per CTA), 128 elements per thread, exactly one shared-memory exchange
-//     per row (conflict-free XOR swizzle), on a balanced contiguous range of rows per SM; each
-//     worker's next row is prefetched with cp.async while the current one is processed, and the
-//     workspace stores rows bit-permuted so that every row access is a contiguous 256-byte span;
+//   * one CTA of 8 warps per SM; a row is one worker's (2^(R-7) threads, 128 elements each):
+//     one round in registers, one conflict-free XOR-swizzled shared-memory exchange, a second
+//     round (plus one warp-shuffle stage for R = 14); each worker's next row is prefetched with
+//     cp.async; rows are spread as balanced contiguous ranges per SM;
+//   * the workspace stores rows bit-permuted (sigma) so that every row access of phases 1 and 3
+//     is one contiguous 256-byte span per warp instruction;
 //   * phase 2 gives columns to threads: whole columns in registers when a column has <= 128
 //     elements; otherwise the two warps (w, w+4) that share a TMEM lane quarter hold one column
-//     per lane (Blackwell tensor memory as per-thread storage, 256 fp32 per thread), trade the
-//     bit between their halves through TMEM, and a 1024-element column adds one shuffle stage;
-//   * column ranges are balanced and aligned to 8 columns (32-byte sectors); for 1024-row columns
-//     the gains are staged through shared memory with cp.async one round-B iteration ahead.
-// Phase 2's flat-index bits are the row bits [13, m); the gain multiplies by G[j*2^13 + c]/L.
+//     per lane (Blackwell tensor memory as per-thread storage, up to 256 fp32 per thread) and
+//     trade the bit between their halves through TMEM;
+//   * column ranges are balanced and aligned to 8 columns (32-byte sectors).
 #pragma once
 
 #include "whtmix_kernels.cuh"
@@ -25,18 +29,25 @@
 namespace whtmix {
 namespace fast {
 
-constexpr int THREADS = 256;   // 8 warps: four 64-thread row workers; warps w, w+4 share TMEM lanes
-constexpr int RB = 13;         // row bits
-constexpr int ROWLEN = 1 << RB;
-constexpr int WORKER = 64;     // threads per row worker
-constexpr int NWORKERS = THREADS / WORKER;
-// shared memory: four row exchange buffers (128 KiB) and four 16 KiB row staging areas for
-// cp.async prefetch of each worker's next row.  More than half an SM, so exactly one CTA per SM.
-constexpr int STAGE_FLOATS = 4096;
-constexpr size_t SMEM_XBUF_BYTES = NWORKERS * ROWLEN * sizeof(float);
-constexpr size_t SMEM_BYTES = SMEM_XBUF_BYTES + NWORKERS * STAGE_FLOATS * sizeof(float);
-static_assert(SMEM_XBUF_BYTES >= 128 * THREADS * sizeof(float), "phase 2 stages 128 gains per thread in the row buffers");
+constexpr int THREADS = 256;  // 8 warps; warps w and w+4 share a TMEM lane quarter
+// shared memory: row exchange buffers (128 KiB) and row staging areas for the cp.async prefetch
+// (64 KiB).  More than half an SM, so exactly one CTA runs per SM.
+constexpr size_t SMEM_XBUF_BYTES = 128 * 1024;
+constexpr size_t SMEM_STAGE_BYTES = 64 * 1024;
+constexpr size_t SMEM_BYTES = SMEM_XBUF_BYTES + SMEM_STAGE_BYTES;
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory per CTA");
+
+// Row geometry for R row bits: 128 elements per thread.
+template <int R>
+struct Row {
+  static constexpr int LEN = 1 << R;
+  static constexpr int WORKER = 1 << (R - 7);          // threads per row
+  static constexpr int NWORKERS = THREADS / WORKER;
+  static constexpr int VSTRIDE = 1 << (R - 4);         // element stride between a thread's 16 vectors
+  static constexpr int STAGE = SMEM_STAGE_BYTES / sizeof(float) / NWORKERS;  // staging floats per worker
+  static_assert(NWORKERS * LEN * sizeof(float) == SMEM_XBUF_BYTES, "one exchange buffer per worker");
+  static_assert(STAGE >= 64 * WORKER, "staging holds 16 bf16 vectors or 32 fp32 pairs per thread");
+};
 
 // ---------------------------------------------------------------------------------------------
 // packed fp32 pairs
@@ -127,28 +138,39 @@ __device__ __forceinline__ void tmem_st16(uint32_t ta, const float (&r)[16]) {
 }
 
 // ---------------------------------------------------------------------------------------------
-// Row exchange buffer: word address of row element r (13 bits), XOR-swizzled so that both access
-// patterns below are bank-conflict free:
+// Row exchange buffer: word address of row element r, XOR-swizzled so that both access patterns
+// below are bank-conflict free:
 //   layout V (16-byte vectors of r0..r1, lanes on r3..r7): bits 2..4 = (r2^r5, r3^r9, r4^r10)
 //   layout P (8-byte pairs of r0, lanes on r1, r2, r9, r10, r11): bits 1..4 = (r1, r2^r5, r3^r9, r4^r10)
 __device__ __forceinline__ int xswz(int r) {
   return r ^ (((r >> 5) & 1) << 2) ^ (((r >> 9) & 1) << 3) ^ (((r >> 10) & 1) << 4);
 }
 
-// Workspace rows are stored with their 13 index bits permuted (sigma), so that layout P's lanes
+// Workspace rows are stored with their index bits permuted (sigma), so that layout P's lanes
 // (r1, r2, r9, r10, r11, plus the in-register pair bit r0) cover 64 consecutive floats: phase 1's
 // stores and phase 3's loads are one 256-byte span per warp instruction.  Storage position s of
-// row element r: s = (r0, r1, r2, r9, r10, r11, r3, r4, r5, r6, r7, r8, r12) from bit 0 up.
+// row element r: s = (r0, r1, r2, r9, r10, r11, r3, r4, r5, r6, r7, r8, r12, r13) from bit 0 up.
 // Phase 2 works in storage positions and maps back to the logical column only to index G.
 __device__ __forceinline__ int sigma(int r) {
-  return (r & 7) | (((r >> 9) & 7) << 3) | (((r >> 3) & 63) << 6) | (r & 4096);
+  return (r & 7) | (((r >> 9) & 7) << 3) | (((r >> 3) & 63) << 6) | (r & ~4095);
 }
 __device__ __forceinline__ int sigma_inv(int s) {
-  return (s & 7) | (((s >> 6) & 63) << 3) | (((s >> 3) & 7) << 9) | (s & 4096);
+  return (s & 7) | (((s >> 6) & 63) << 3) | (((s >> 3) & 7) << 9) | (s & ~4095);
 }
 
+template <int R>
 __device__ __forceinline__ void worker_sync(int worker) {
-  asm volatile("bar.sync %0, %1;" ::"r"(worker + 1), "r"(WORKER) : "memory");
+  asm volatile("bar.sync %0, %1;" ::"r"(worker + 1), "r"(Row<R>::WORKER) : "memory");
+}
+
+// Butterfly on a row bit held by lane bit 2 (r9 in layout P when R = 14): lane pairs (l, l ^ 4).
+__device__ __forceinline__ void bfly_lane4(float2 (&b)[64]) {
+  const float2 sgn = (threadIdx.x & 4) ? make_float2(-1.f, -1.f) : make_float2(1.f, 1.f);
+#pragma unroll
+  for (int s = 0; s < 64; ++s) {
+    const float2 p = make_float2(__shfl_xor_sync(0xffffffffu, b[s].x, 4), __shfl_xor_sync(0xffffffffu, b[s].y, 4));
+    b[s] = fma2(b[s], sgn, p);
+  }
 }
 
 // Storage <-> fp32 for the two floating dtypes.
@@ -205,54 +227,76 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // Row prefetch.  Every thread copies exactly the 16-byte (8-byte) chunks it will read back
-// itself, so the staging area needs no barrier; chunk k of thread wt sits at (k * 64 + wt), which
-// makes each warp's read-back one contiguous 512-byte (256-byte) span.
+// itself, so the staging area needs no barrier; chunk k of thread wt sits at (k * WORKER + wt),
+// which makes each warp's read-back one contiguous span.
 // Phase 1 stages a whole bf16 row (16 vectors of 8 elements) or the first half of an fp32 row.
-template <int D>
+template <int D, int R>
 __device__ __forceinline__ void stage_row_in(const void* src, long long e0, float* stg, int wt) {
+  constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   if constexpr (D == DT_BF16) {
 #pragma unroll
     for (int v = 0; v < 16; ++v)
-      cp_async16(stg + (v * 64 + wt) * 4, static_cast<const unsigned short*>(src) + e0 + 8 * wt + 512 * v);
+      cp_async16(stg + (v * WK + wt) * 4, static_cast<const unsigned short*>(src) + e0 + 8 * wt + VS * v);
   } else {
 #pragma unroll
     for (int v = 0; v < 8; ++v)
 #pragma unroll
       for (int h2 = 0; h2 < 2; ++h2)
-        cp_async16(stg + ((2 * v + h2) * 64 + wt) * 4, static_cast<const float*>(src) + e0 + 8 * wt + 512 * v + 4 * h2);
+        cp_async16(stg + ((2 * v + h2) * WK + wt) * 4, static_cast<const float*>(src) + e0 + 8 * wt + VS * v + 4 * h2);
   }
   cp_async_commit();
 }
 // Phase 3 stages the first 32 of the 64 pairs each thread reads in layout P.
 __device__ __forceinline__ int pbase_of(int wt) { return 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2); }
+template <int R>
 __device__ __forceinline__ void stage_row_out(const float* src_ws, float* stg, int wt) {
   const int pbase = pbase_of(wt);
 #pragma unroll
-  for (int s = 0; s < 32; ++s) cp_async8(stg + (s * 64 + wt) * 2, src_ws + sigma(pbase + 8 * s));
+  for (int s = 0; s < 32; ++s) cp_async8(stg + (s * Row<R>::WORKER + wt) * 2, src_ws + sigma(pbase + 8 * s));
   cp_async_commit();
 }
 
+// round over the layout-V register bits: r1, r2 (inside a vector) and the 4 vector bits
+__device__ __forceinline__ void round_v(float2 (&a)[16][4]) {
+#pragma unroll
+  for (int v = 0; v < 16; ++v) {
+    bf2(a[v][0], a[v][1]);
+    bf2(a[v][2], a[v][3]);
+    bf2(a[v][0], a[v][2]);
+    bf2(a[v][1], a[v][3]);
+  }
+#pragma unroll
+  for (int h = 1; h < 16; h <<= 1)
+#pragma unroll
+    for (int v = 0; v < 16; ++v)
+      if ((v & h) == 0)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
+}
+
 // ---------------------------------------------------------------------------------------------
-// Phase 1 row: X (dtype D) -> workspace (fp32), butterflies on all 13 row bits.
-//   layout V: thread wt holds r0..r2 (8-vectors) x r9..r12 (16 vectors); wt = r3..r8.
-//     round A: bits r1, r2, r9..r12 (pairs on r0).
-//   exchange through smem, then layout P: thread holds pairs (r0) x r3..r8; wt bits =
-//     (r1, r2, r9, r10, r11, r12).  round B: r0 (inside the pairs) and r3..r8.
+// Phase 1 row: X (dtype D) -> workspace (fp32), butterflies on all R row bits.
+//   layout V: thread wt holds r0..r2 (8-vectors) x 16 vectors (bits R-4..R-1); wt = r3..r(R-5).
+//     round A: bits r1, r2 and the vector bits (pairs on r0).
+//   exchange through smem, then layout P: thread holds pairs (r0) x r3..r8; wt bits = (r1, r2,
+//     r9, ...) with lanes on (r1, r2, r9, r10, r11).  round B: r0 (inside the pairs), r3..r8,
+//     and for R = 14 r9 by one shuffle stage.
 // The row arrives through the staging area (prefetched while the previous row was processed);
 // the next row's prefetch (e0_next >= 0) is issued as soon as this row is in registers.
-template <int D>
+template <int D, int R>
 __device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, float* stg,
                                                int wt, int worker, long long e0_next) {
-  float2 a[16][4];  // [v = r9..r12][r1 + 2 r2]
+  constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
+  float2 a[16][4];  // [vector][r1 + 2 r2]
   if constexpr (D == DT_F32) {
 #pragma unroll
-    for (int v = 8; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + 512 * v, a[v]);
+    for (int v = 8; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + VS * v, a[v]);
   }
   cp_async_wait_all();
   if constexpr (D == DT_BF16) {
 #pragma unroll
     for (int v = 0; v < 16; ++v) {
-      const uint4 u = *reinterpret_cast<const uint4*>(stg + (v * 64 + wt) * 4);
+      const uint4 u = *reinterpret_cast<const uint4*>(stg + (v * WK + wt) * 4);
       const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
       for (int i = 0; i < 4; ++i) a[v][i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
@@ -260,145 +304,125 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
   } else {
 #pragma unroll
     for (int v = 0; v < 8; ++v) {
-      const float4 q0 = *reinterpret_cast<const float4*>(stg + ((2 * v) * 64 + wt) * 4);
-      const float4 q1 = *reinterpret_cast<const float4*>(stg + ((2 * v + 1) * 64 + wt) * 4);
+      const float4 q0 = *reinterpret_cast<const float4*>(stg + ((2 * v) * WK + wt) * 4);
+      const float4 q1 = *reinterpret_cast<const float4*>(stg + ((2 * v + 1) * WK + wt) * 4);
       a[v][0] = make_float2(q0.x, q0.y);
       a[v][1] = make_float2(q0.z, q0.w);
       a[v][2] = make_float2(q1.x, q1.y);
       a[v][3] = make_float2(q1.z, q1.w);
     }
   }
-  // round A
-#pragma unroll
-  for (int v = 0; v < 16; ++v) {
-    bf2(a[v][0], a[v][1]);
-    bf2(a[v][2], a[v][3]);
-    bf2(a[v][0], a[v][2]);
-    bf2(a[v][1], a[v][3]);
-  }
-#pragma unroll
-  for (int h = 1; h < 16; h <<= 1)
-#pragma unroll
-    for (int v = 0; v < 16; ++v)
-      if ((v & h) == 0)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
-  if (e0_next >= 0) stage_row_in<D>(src, e0_next, stg, wt);
+  round_v(a);
+  if (e0_next >= 0) stage_row_in<D, R>(src, e0_next, stg, wt);
   // exchange V -> P
 #pragma unroll
   for (int v = 0; v < 16; ++v)
 #pragma unroll
     for (int r2 = 0; r2 < 2; ++r2) {
-      const int r = 8 * wt + 512 * v + 4 * r2;
+      const int r = 8 * wt + VS * v + 4 * r2;
       *reinterpret_cast<float4*>(xbuf + xswz(r)) = make_float4(a[v][2 * r2].x, a[v][2 * r2].y, a[v][2 * r2 + 1].x, a[v][2 * r2 + 1].y);
     }
-  worker_sync(worker);
-  const int pbase = pbase_of(wt);  // r1, r2, r9..r12
+  worker_sync<R>(worker);
+  const int pbase = pbase_of(wt);
   float2 b[64];  // [s = r3..r8]
 #pragma unroll
   for (int s = 0; s < 64; ++s) b[s] = *reinterpret_cast<const float2*>(xbuf + xswz(pbase + 8 * s));
-  worker_sync(worker);  // buffer free for the next row
+  worker_sync<R>(worker);  // buffer free for the next row
   // round B
 #pragma unroll
   for (int s = 0; s < 64; ++s) bf_in(b[s]);
   bfly_all<64>(b);
+  if constexpr (R == 14) bfly_lane4(b);
 #pragma unroll
   for (int s = 0; s < 64; ++s) __stcg(reinterpret_cast<float2*>(dst_ws + sigma(pbase + 8 * s)), b[s]);
 }
 
-// Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all 13 row bits (mirror of phase 1).
+// Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all R row bits (mirror of phase 1).
 // The first half of the row's pairs arrives through the staging area; src_next (if not null) is
 // the next row, whose prefetch is issued once this row is in registers.
-template <int D>
+template <int D, int R>
 __device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, float* xbuf, float* stg,
                                                 int wt, int worker, const float* src_next) {
+  constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   const int pbase = pbase_of(wt);
   float2 b[64];
 #pragma unroll
   for (int s = 32; s < 64; ++s) b[s] = __ldcg(reinterpret_cast<const float2*>(src_ws + sigma(pbase + 8 * s)));
   cp_async_wait_all();
 #pragma unroll
-  for (int s = 0; s < 32; ++s) b[s] = *reinterpret_cast<const float2*>(stg + (s * 64 + wt) * 2);
-  bfly_all<64>(b);  // round A: r3..r8
-  if (src_next != nullptr) stage_row_out(src_next, stg, wt);
+  for (int s = 0; s < 32; ++s) b[s] = *reinterpret_cast<const float2*>(stg + (s * WK + wt) * 2);
+  bfly_all<64>(b);  // round A: r3..r8 (and r9 for R = 14)
+  if constexpr (R == 14) bfly_lane4(b);
+  if (src_next != nullptr) stage_row_out<R>(src_next, stg, wt);
 #pragma unroll
   for (int s = 0; s < 64; ++s) *reinterpret_cast<float2*>(xbuf + xswz(pbase + 8 * s)) = b[s];
-  worker_sync(worker);
+  worker_sync<R>(worker);
   float2 a[16][4];
 #pragma unroll
   for (int v = 0; v < 16; ++v)
 #pragma unroll
     for (int r2 = 0; r2 < 2; ++r2) {
-      const float4 q = *reinterpret_cast<const float4*>(xbuf + xswz(8 * wt + 512 * v + 4 * r2));
+      const float4 q = *reinterpret_cast<const float4*>(xbuf + xswz(8 * wt + VS * v + 4 * r2));
       a[v][2 * r2] = make_float2(q.x, q.y);
       a[v][2 * r2 + 1] = make_float2(q.z, q.w);
     }
-  worker_sync(worker);
-  // round B: r0, r1, r2, r9..r12
+  worker_sync<R>(worker);
+  // round B: r0, r1, r2 and the vector bits
 #pragma unroll
-  for (int v = 0; v < 16; ++v) {
+  for (int v = 0; v < 16; ++v)
 #pragma unroll
     for (int i = 0; i < 4; ++i) bf_in(a[v][i]);
-    bf2(a[v][0], a[v][1]);
-    bf2(a[v][2], a[v][3]);
-    bf2(a[v][0], a[v][2]);
-    bf2(a[v][1], a[v][3]);
-  }
+  round_v(a);
 #pragma unroll
-  for (int h = 1; h < 16; h <<= 1)
-#pragma unroll
-    for (int v = 0; v < 16; ++v)
-      if ((v & h) == 0)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) bf2(a[v][i], a[v + h][i]);
-#pragma unroll
-  for (int v = 0; v < 16; ++v) IOv<D>::st8(dst, e0 + 8 * wt + 512 * v, a[v]);
+  for (int v = 0; v < 16; ++v) IOv<D>::st8(dst, e0 + 8 * wt + VS * v, a[v]);
 }
 
 // ---------------------------------------------------------------------------------------------
-// Phase 2, register variant (Q <= 6): a thread owns two adjacent columns (one pair) x 2^Q rows.
-template <int Q>
+// Phase 2, register variant (Q <= 6): a thread owns two adjacent storage positions (one logical
+// column pair) x 2^Q rows.
+template <int Q, int R>
 __device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
-  constexpr int R = 1 << Q;
+  constexpr int NR = 1 << Q;
   const float2 sc = make_float2(scale, scale);
   for (long long u0 = u_begin; u0 < u_end; u0 += 2 * THREADS) {
     const long long u = u0 + 2 * threadIdx.x;  // even: the pair never straddles a plane
     if (u >= u_end) break;
-    const long long b = u >> RB;
-    const int sp = static_cast<int>(u & (ROWLEN - 1));  // storage position (even); sp + 1 is column c + 1
+    const long long b = u >> R;
+    const int sp = static_cast<int>(u & ((1 << R) - 1));  // storage position (even); sp + 1 is column c + 1
     float* base = ws + (b << m) + sp;
     const float* gb = g + sigma_inv(sp);
-    float2 v[R];
+    float2 v[NR];
 #pragma unroll
-    for (int j = 0; j < R; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << RB)));
-    bfly_all<R>(v);
+    for (int j = 0; j < NR; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << R)));
+    bfly_all<NR>(v);
 #pragma unroll
-    for (int j = 0; j < R; ++j) v[j] = mul2(v[j], mul2(__ldg(reinterpret_cast<const float2*>(gb + (static_cast<long long>(j) << RB))), sc));
-    bfly_all<R>(v);
+    for (int j = 0; j < NR; ++j) v[j] = mul2(v[j], mul2(__ldg(reinterpret_cast<const float2*>(gb + (static_cast<long long>(j) << R))), sc));
+    bfly_all<NR>(v);
 #pragma unroll
-    for (int j = 0; j < R; ++j) __stcg(reinterpret_cast<float2*>(base + (static_cast<long long>(j) << RB)), v[j]);
+    for (int j = 0; j < NR; ++j) __stcg(reinterpret_cast<float2*>(base + (static_cast<long long>(j) << R)), v[j]);
   }
 }
 
 // Phase 2, register variant for Q = 7: a thread owns one column of 128 rows as 64 pairs (j, j + 64).
+template <int R>
 __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
   for (long long u0 = u_begin; u0 < u_end; u0 += THREADS) {
     const long long u = u0 + threadIdx.x;
     if (u >= u_end) break;
-    const long long b = u >> RB;
-    const int sp = static_cast<int>(u & (ROWLEN - 1));
+    const long long b = u >> R;
+    const int sp = static_cast<int>(u & ((1 << R) - 1));
     float* base = ws + (b << m) + sp;
     const float* gb = g + sigma_inv(sp);
     float2 v[64];
 #pragma unroll
     for (int j = 0; j < 64; ++j)
-      v[j] = make_float2(__ldcg(base + (static_cast<long long>(j) << RB)), __ldcg(base + (static_cast<long long>(j + 64) << RB)));
+      v[j] = make_float2(__ldcg(base + (static_cast<long long>(j) << R)), __ldcg(base + (static_cast<long long>(j + 64) << R)));
     bfly_all<64>(v);
 #pragma unroll
     for (int j = 0; j < 64; ++j) bf_in(v[j]);
 #pragma unroll
     for (int j = 0; j < 64; ++j) {
-      const float2 gg = make_float2(__ldg(gb + (static_cast<long long>(j) << RB)), __ldg(gb + (static_cast<long long>(j + 64) << RB)));
+      const float2 gg = make_float2(__ldg(gb + (static_cast<long long>(j) << R)), __ldg(gb + (static_cast<long long>(j + 64) << R)));
       v[j] = mul2(v[j], mul2(gg, make_float2(scale, scale)));
     }
 #pragma unroll
@@ -406,8 +430,8 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
     bfly_all<64>(v);
 #pragma unroll
     for (int j = 0; j < 64; ++j) {
-      __stcg(base + (static_cast<long long>(j) << RB), v[j].x);
-      __stcg(base + (static_cast<long long>(j + 64) << RB), v[j].y);
+      __stcg(base + (static_cast<long long>(j) << R), v[j].x);
+      __stcg(base + (static_cast<long long>(j + 64) << R), v[j].y);
     }
   }
 }
@@ -417,65 +441,39 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
 __device__ __forceinline__ void pair_sync(int quarter) {
   tmem_wait_st();
   tmem_fence_before();
-  asm volatile("bar.sync %0, %1;" ::"r"(NWORKERS + 1 + quarter), "r"(64) : "memory");
+  asm volatile("bar.sync %0, %1;" ::"r"(5 + quarter), "r"(64) : "memory");
   tmem_fence_after();
 }
 
-// Phase 2, TMEM variant (8 <= Q <= 10).  Per TMEM lane: one column half of Eh = 2^(Q - lanebit)
-// rows; the lane's 2*Et columns hold element k of warp half hw at column hw*Et + k (Et = Eh/2
-// elements per thread).  Bits: k0..k(et-1) local to a thread, k(et) = warp half (traded through
-// TMEM), and for Q = 10 the top row bit = lane bit 4 (one shuffle stage).
-//   round A: own Et elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
-//   round B: bits k6..k(et) (+ lane bit) forward, gain, back; each warp half takes k5 = hw
-//   round C: own Et elements, bits k0..k5 again, TMEM -> global
-//   G for round B is staged in shared memory (gstage, the idle row buffers) with cp.async, one
-//   round-B iteration ahead: value v of thread t sits at gstage[v * THREADS + t], and every thread
-//   reads back only what it copied itself, so no barrier is needed.
-template <int Q>
+// Phase 2, TMEM variant (Q = 8, 9).  Per TMEM lane: one column of 2^Q rows; the lane's 2*ET
+// columns hold element k of warp half hw at column hw*ET + k (ET = 2^(Q-1) elements per thread).
+// Bits: k0..k(et-1) local to a thread, k(et) = warp half (traded through TMEM).
+//   round A: own ET elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
+//   round B: bits k6..k(et) forward, gain, back; each warp half takes k5 = hw
+//   round C: own ET elements, bits k0..k5 again, TMEM -> global
+template <int Q, int R>
 __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float scale, int m, long long u_begin,
-                                              long long u_end, uint32_t tlane, float* gstage) {
-  constexpr bool LANEBIT = Q == 10;
-  constexpr int ET_BITS = Q - 1 - (LANEBIT ? 1 : 0);  // 8, 8, 7 for Q = 10, 9, 8
+                                              long long u_end, uint32_t tlane) {
+  constexpr int ET_BITS = Q - 1;                       // 8, 7 for Q = 9, 8
   constexpr int ET = 1 << ET_BITS;
-  constexpr int PER_PASS = LANEBIT ? 64 : 128;         // columns per pass
+  constexpr int PER_PASS = 128;                        // columns per pass (one per TMEM lane)
   constexpr int ITA = ET / 128;                        // round A/C iterations (64 pairs each)
   constexpr int NH = 1 << (ET_BITS - 5);               // high combinations in round B (incl. warp half)
   constexpr int W = 64 / NH;                           // pairs per high combination
   constexpr int ITB = 16 / W;                          // round B iterations
-  // With the shuffle stages in round B there are no spare registers to hoist the G loads above
-  // them, so for Q = 10 G is staged ahead through shared memory; otherwise it is loaded directly.
-  constexpr bool STAGE_G = LANEBIT;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int quarter = warp & 3, hw = warp >> 2;
-  const int slot = LANEBIT ? quarter * 16 + (lane & 15) : quarter * 32 + lane;
-  const int h = LANEBIT ? (lane >> 4) : 0;
-  const float2 sgn = h ? make_float2(-1.f, -1.f) : make_float2(1.f, 1.f);
+  const int slot = quarter * 32 + lane;
   const float2 sc = make_float2(scale, scale);
   for (long long u0 = u_begin; u0 < u_end; u0 += PER_PASS) {
     const long long u = u0 + slot;
     const bool active = u < u_end;
     const long long uu = active ? u : u_begin;  // inactive lanes compute on a valid column, never store
-    const long long b = uu >> RB;
-    const int sp = static_cast<int>(uu & (ROWLEN - 1));  // storage position of the column
-    float* colp = ws + (b << m) + sp + (static_cast<long long>(h) << (9 + RB));
-    const float* gcol = g + sigma_inv(sp) + (static_cast<long long>(h) << (9 + RB));
-    float* own = colp + (static_cast<long long>(hw * ET) << RB);
-    // G rows of round-B iteration `it`, in the order the gain step consumes them
-    auto stage_gain = [&](int it) {
-#pragma unroll
-      for (int s = 0; s < NH; ++s) {
-        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
-#pragma unroll
-        for (int w = 0; w < W; ++w) {
-          const int vi = 2 * (s * W + w);
-          cp_async4(gstage + vi * THREADS + threadIdx.x, gcol + ((j0 + 2 * w) << RB));
-          cp_async4(gstage + (vi + 1) * THREADS + threadIdx.x, gcol + ((j0 + 2 * w + 1) << RB));
-        }
-      }
-      cp_async_commit();
-    };
-    if constexpr (STAGE_G) stage_gain(0);
+    const long long b = uu >> R;
+    const int sp = static_cast<int>(uu & ((1 << R) - 1));  // storage position of the column
+    float* colp = ws + (b << m) + sp;
+    const float* gcol = g + sigma_inv(sp);
+    float* own = colp + (static_cast<long long>(hw * ET) << R);
     // round A
 #pragma unroll 1
     for (int it = 0; it < ITA; ++it) {
@@ -483,7 +481,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 #pragma unroll
       for (int k = 0; k < 64; ++k) {
         const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
-        v[k] = make_float2(__ldcg(own + (k0 << RB)), __ldcg(own + (k1 << RB)));
+        v[k] = make_float2(__ldcg(own + (k0 << R)), __ldcg(own + (k1 << R)));
       }
       bfly_all<64>(v);
 #pragma unroll
@@ -523,47 +521,16 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
           if ((s & hh) == 0)
 #pragma unroll
             for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
-      if (LANEBIT) {
 #pragma unroll
-        for (int s = 0; s < NH; ++s)
+      for (int s = 0; s < NH; ++s) {
+        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
 #pragma unroll
-          for (int w = 0; w < W; ++w) {
-            const float2 p = make_float2(__shfl_xor_sync(0xffffffffu, v[s][w].x, 16), __shfl_xor_sync(0xffffffffu, v[s][w].y, 16));
-            v[s][w] = fma2(v[s][w], sgn, p);
-          }
-      }
-      if constexpr (STAGE_G) {
-        cp_async_wait_all();
-#pragma unroll
-        for (int s = 0; s < NH; ++s)
-#pragma unroll
-          for (int w = 0; w < W; ++w) {
-            const int vi = 2 * (s * W + w);
-            const float2 gg = make_float2(gstage[vi * THREADS + threadIdx.x], gstage[(vi + 1) * THREADS + threadIdx.x]);
-            v[s][w] = mul2(v[s][w], mul2(gg, sc));
-          }
-        if (it + 1 < ITB) stage_gain(it + 1);
-      } else {
-#pragma unroll
-        for (int s = 0; s < NH; ++s) {
-          const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-          const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
-#pragma unroll
-          for (int w = 0; w < W; ++w) {
-            const long long j = j0 + 2 * w;
-            const float2 gg = make_float2(__ldg(gcol + (j << RB)), __ldg(gcol + ((j + 1) << RB)));
-            v[s][w] = mul2(v[s][w], mul2(gg, sc));
-          }
+        for (int w = 0; w < W; ++w) {
+          const long long j = j0 + 2 * w;
+          const float2 gg = make_float2(__ldg(gcol + (j << R)), __ldg(gcol + ((j + 1) << R)));
+          v[s][w] = mul2(v[s][w], mul2(gg, sc));
         }
-      }
-      if (LANEBIT) {
-#pragma unroll
-        for (int s = 0; s < NH; ++s)
-#pragma unroll
-          for (int w = 0; w < W; ++w) {
-            const float2 p = make_float2(__shfl_xor_sync(0xffffffffu, v[s][w].x, 16), __shfl_xor_sync(0xffffffffu, v[s][w].y, 16));
-            v[s][w] = fma2(v[s][w], sgn, p);
-          }
       }
 #pragma unroll
       for (int hh = 1; hh < NH; hh <<= 1)
@@ -607,8 +574,8 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 #pragma unroll
         for (int k = 0; k < 64; ++k) {
           const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
-          __stcg(own + (k0 << RB), v[k].x);
-          __stcg(own + (k1 << RB), v[k].y);
+          __stcg(own + (k0 << R), v[k].x);
+          __stcg(own + (k1 << R), v[k].y);
         }
       }
     }
@@ -619,20 +586,22 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 
 // ---------------------------------------------------------------------------------------------
 // Forward kernel: persistent cooperative grid (one CTA per SM), plane groups of P.gp planes,
-// three phases.  Q = m - 13 is a template parameter so that every register array has a static size.
-template <int D, int Q>
+// three phases.  R and Q are template parameters so that every register array has a static size.
+template <int D, int R, int Q>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
+  static_assert((R == 13 && Q >= 1 && Q <= 8) || (R == 14 && (Q == 8 || Q == 9)), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   __shared__ uint32_t tmem_slot;
   constexpr bool USE_TMEM = Q >= 8;
-  float* xbuf_all = reinterpret_cast<float*>(smem_raw);
-  const int worker = threadIdx.x / WORKER, wt = threadIdx.x % WORKER;
-  float* xbuf = xbuf_all + worker * ROWLEN;
-  float* stg = xbuf_all + NWORKERS * ROWLEN + worker * STAGE_FLOATS;
+  using RW = Row<R>;
+  float* sm = reinterpret_cast<float*>(smem_raw);
+  const int worker = threadIdx.x / RW::WORKER, wt = threadIdx.x % RW::WORKER;
+  float* xbuf = sm + worker * RW::LEN;
+  float* stg = sm + SMEM_XBUF_BYTES / sizeof(float) + worker * RW::STAGE;
   float* ws = static_cast<float*>(P.ws);
   const float* g = static_cast<const float*>(P.g);
-  const int m = RB + Q;
+  const int m = R + Q;
   uint32_t tlane = 0;
   if constexpr (USE_TMEM) {
     if (threadIdx.x < 32) tmem_alloc_512(&tmem_slot);
@@ -646,28 +615,28 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     const long long rows = nb << Q;
     const long long rb = rows * blockIdx.x / gridDim.x, re = rows * (blockIdx.x + 1) / gridDim.x;
     // phase-2 column range: balanced, aligned to 8 columns
-    const long long cols = nb << RB;
+    const long long cols = nb << R;
     const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
     const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
     // phase 1: X -> ws, row bits
-    if (rb + worker < re) stage_row_in<D>(P.x, (b0 << m) + ((rb + worker) << RB), stg, wt);
-    for (long long r = rb + worker; r < re; r += NWORKERS) {
-      const long long rn = r + NWORKERS;
-      row_forward_in<D>(P.x, (b0 << m) + (r << RB), ws + (r << RB), xbuf, stg, wt, worker,
-                        rn < re ? (b0 << m) + (rn << RB) : -1);
+    if (rb + worker < re) stage_row_in<D, R>(P.x, (b0 << m) + ((rb + worker) << R), stg, wt);
+    for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
+      const long long rn = r + RW::NWORKERS;
+      row_forward_in<D, R>(P.x, (b0 << m) + (r << R), ws + (r << R), xbuf, stg, wt, worker,
+                           rn < re ? (b0 << m) + (rn << R) : -1);
     }
     if (!grid_sync(P.bar, &flag)) break;
     // phase 2: column bits, gain, column bits
-    if constexpr (USE_TMEM) col_pass_tmem<Q>(ws, g, P.scale, m, cb, ce, tlane, xbuf_all);
-    else if constexpr (Q == 7) col_pass_single128(ws, g, P.scale, m, cb, ce);
-    else col_pass_pairs<Q>(ws, g, P.scale, m, cb, ce);
+    if constexpr (USE_TMEM) col_pass_tmem<Q, R>(ws, g, P.scale, m, cb, ce, tlane);
+    else if constexpr (Q == 7) col_pass_single128<R>(ws, g, P.scale, m, cb, ce);
+    else col_pass_pairs<Q, R>(ws, g, P.scale, m, cb, ce);
     if (!grid_sync(P.bar, &flag)) break;
     // phase 3: ws -> Y, row bits
-    if (rb + worker < re) stage_row_out(ws + ((rb + worker) << RB), stg, wt);
-    for (long long r = rb + worker; r < re; r += NWORKERS) {
-      const long long rn = r + NWORKERS;
-      row_forward_out<D>(ws + (r << RB), P.y, (b0 << m) + (r << RB), xbuf, stg, wt, worker,
-                         rn < re ? ws + (rn << RB) : nullptr);
+    if (rb + worker < re) stage_row_out<R>(ws + ((rb + worker) << R), stg, wt);
+    for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
+      const long long rn = r + RW::NWORKERS;
+      row_forward_out<D, R>(ws + (r << R), P.y, (b0 << m) + (r << R), xbuf, stg, wt, worker,
+                            rn < re ? ws + (rn << R) : nullptr);
     }
     if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) break;
   }

@@ -39,10 +39,10 @@ inline cudaError_t occupancy_cached(const void* kernel, size_t smem, int* occ) {
 // Every variant requests more than half an SM's shared memory, so exactly one CTA runs per SM:
 // two CTAs on one SM would both ask for all 512 TMEM columns, and the second would wait in
 // tcgen05.alloc while the first waits for it at the device-wide barrier.
-template <int D, int Q>
+template <int D, int R, int Q>
 cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
   const size_t smem = SMEM_BYTES;
-  const void* k = reinterpret_cast<const void*>(k_forward_fast<D, Q>);
+  const void* k = reinterpret_cast<const void*>(k_forward_fast<D, R, Q>);
   int occ = 0;
   cudaError_t e = occupancy_cached(k, smem, &occ);
   if (e != cudaSuccess) return e;
@@ -52,19 +52,21 @@ cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
   return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, smem, stream);
 }
 
+// Rows of 2^13 elements up to 2^21-element planes; rows of 2^14 for 2^22 and 2^23 (columns of
+// at most 512 rows).
 template <int D>
 cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
-  switch (P.m - RB) {
-    case 1: return launch_one<D, 1>(P, sms, stream);
-    case 2: return launch_one<D, 2>(P, sms, stream);
-    case 3: return launch_one<D, 3>(P, sms, stream);
-    case 4: return launch_one<D, 4>(P, sms, stream);
-    case 5: return launch_one<D, 5>(P, sms, stream);
-    case 6: return launch_one<D, 6>(P, sms, stream);
-    case 7: return launch_one<D, 7>(P, sms, stream);
-    case 8: return launch_one<D, 8>(P, sms, stream);
-    case 9: return launch_one<D, 9>(P, sms, stream);
-    case 10: return launch_one<D, 10>(P, sms, stream);
+  switch (P.m) {
+    case 14: return launch_one<D, 13, 1>(P, sms, stream);
+    case 15: return launch_one<D, 13, 2>(P, sms, stream);
+    case 16: return launch_one<D, 13, 3>(P, sms, stream);
+    case 17: return launch_one<D, 13, 4>(P, sms, stream);
+    case 18: return launch_one<D, 13, 5>(P, sms, stream);
+    case 19: return launch_one<D, 13, 6>(P, sms, stream);
+    case 20: return launch_one<D, 13, 7>(P, sms, stream);
+    case 21: return launch_one<D, 13, 8>(P, sms, stream);
+    case 22: return launch_one<D, 14, 8>(P, sms, stream);
+    case 23: return launch_one<D, 14, 9>(P, sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }
