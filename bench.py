@@ -47,7 +47,7 @@ def kernel_name(w) -> str:
     """The kernel one whtmix_forward call launches for this workload (mirrors the C ABI's dispatch)."""
     m = (w.N * w.C).bit_length() - 1
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
-        r = 14 if m >= 22 else 13
+        r = 14 if m == 23 else 13
         return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}>"
     return "k_forward_s" if m <= 13 else "k_forward_m"
 

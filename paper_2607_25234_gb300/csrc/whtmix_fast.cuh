@@ -5,7 +5,7 @@
 // for the instruction and latency budget of the path: the butterflies need 2 log2(NC) fp32 adds
 // per element, which at N*C = 2^23 on 152 SMs is about as long as streaming X, G and Y through
 // HBM.  A plane of 2^m elements is viewed as 2^Q rows of 2^R contiguous elements (R = 13, or 14
-// for m >= 22, so that Q <= 9):
+// for m = 23, so that Q <= 9):
 //   phase 1  every row: its R bits forward                              X  -> workspace
 //   phase 2  every column: its Q bits forward, gain G/L, Q bits again   workspace -> workspace
 //   phase 3  every row: its R bits again                                workspace -> Y
@@ -589,7 +589,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 // three phases.  R and Q are template parameters so that every register array has a static size.
 template <int D, int R, int Q>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
-  static_assert((R == 13 && Q >= 1 && Q <= 8) || (R == 14 && (Q == 8 || Q == 9)), "supported row/column split");
+  static_assert((R == 13 && Q >= 1 && Q <= 9) || (R == 14 && Q == 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   __shared__ uint32_t tmem_slot;
