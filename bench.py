@@ -130,18 +130,22 @@ class ClockSampler:
 
 
 def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
-    """Median wall time of the CPU oracle's forward on one [n_tokens, C] plane of the workload."""
+    """Median wall time of the CPU oracle on one [n_tokens, C] plane of the workload: the forward,
+    plus the backward for a training-step workload."""
     import numpy as np
     import oracle
     d = inputs.make_inputs(1, n_tokens, w.C, w.dtype, seed=0,
-                           n_valid=None if w.n_valid is None else min(w.n_valid, n_tokens))
+                           n_valid=None if w.n_valid is None else min(w.n_valid, n_tokens), with_dy=w.backward)
     x = inputs.as_float64(d["x"], w.dtype)
     g = d["g"].astype(np.float64)
+    dy = inputs.as_float64(d["dy"], w.dtype) if w.backward else None
     oracle.forward(x[:, :8, :], g[:8, :])  # load / compile outside the timing
     times = []
     for _ in range(reps):
         t = time.perf_counter()
         oracle.forward(x, g)
+        if dy is not None:
+            oracle.backward(x, g, dy)
         times.append(time.perf_counter() - t)
     return statistics.median(times), times
 
@@ -220,22 +224,42 @@ def ours(args, w):
     g_host = torch.from_numpy(d["g"])
     x0 = x_host.to(dev)
     g0 = g_host.to(dev)
-    set_bytes = x0.numel() * x0.element_size() * 2 + g0.numel() * g0.element_size()
+    # a training step (forward + backward) also reads dY and writes dX and dG
+    dy_host = None
+    if w.backward:
+        dy_host = torch.from_numpy(d["dy"].view(np.int16) if w.dtype == "bf16" else d["dy"])
+        if w.dtype == "bf16":
+            dy_host = dy_host.view(torch.bfloat16)
+    plane_b = x0.numel() * x0.element_size()
+    g_b = g0.numel() * g0.element_size()
+    set_bytes = 2 * plane_b + g_b + ((2 * plane_b + g_b) if w.backward else 0)
     nsets = max(2, -(-3 * l2 // set_bytes))
     xs = [x0] + [x0.clone() for _ in range(nsets - 1)]
     gs = [g0] + [g0.clone() for _ in range(nsets - 1)]
     ys = [torch.empty_like(x0) for _ in range(nsets)]
+    if w.backward:
+        dys = [dy_host.to(dev) for _ in range(nsets)]
+        dxs = [torch.empty_like(x0) for _ in range(nsets)]
+        dgs = [torch.empty_like(g0) for _ in range(nsets)]
     code = whtmix.DTYPE_CODE[tdt]
     stream = torch.cuda.current_stream(dev)
     sp = int(stream.cuda_stream)
     args_c = [(xs[i].data_ptr(), gs[i].data_ptr(), ys[i].data_ptr()) for i in range(nsets)]
+    bargs_c = [(dys[i].data_ptr(), dxs[i].data_ptr(), dgs[i].data_ptr()) for i in range(nsets)] if w.backward else None
     fwd = lib.whtmix_forward
+    bwd = lib.whtmix_backward
+    launches_per_step = 2 if w.backward else 1
 
     def step(i):
         a = args_c[i % nsets]
         rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
         if rc != 0:
             raise whtmix.WhtmixError(rc, "whtmix_forward")
+        if w.backward:
+            bb = bargs_c[i % nsets]
+            rc = bwd(a[0], a[1], bb[0], bb[1], bb[2], w.B, w.N, w.C, code, sp)
+            if rc != 0:
+                raise whtmix.WhtmixError(rc, "whtmix_backward")
 
     # warm-up (also allocates the cached workspace on this stream)
     for i in range(max(args.warmup, 3)):
@@ -285,7 +309,7 @@ def ours(args, w):
     tokens_per_step = w.B * w.N
     value = world * tokens_per_step * K / (elapsed_ms / 1e3)
     kern_mean_ms = statistics.mean(kern_ms)
-    ideal = w.ideal_bytes(backward=False)
+    ideal = w.ideal_bytes()
     peak, peak_kind = measured_peaks()
     achieved = ideal / (kern_mean_ms / 1e3) / 1e9
 
@@ -296,26 +320,38 @@ def ours(args, w):
         gh = g_host.pin_memory()
         yh = torch.empty_like(xh).pin_memory()
         xd, gd, yd = xs[0], gs[0], ys[0]
+        h2d = [(xd, xh), (gd, gh)]
+        d2h = [(yh, yd)]
+        if w.backward:
+            dyh = dy_host.pin_memory()
+            dxh = torch.empty_like(dyh).pin_memory()
+            dgh = torch.empty_like(gh).pin_memory()
+            h2d.append((dys[0], dyh))
+            d2h += [(dxh, dxs[0]), (dgh, dgs[0])]
         ke = max(3, min(K, 50))
-        for _ in range(3):
-            xd.copy_(xh, non_blocking=True)
-            gd.copy_(gh, non_blocking=True)
+
+        def e2e_step():
+            for dst, src in h2d:
+                dst.copy_(src, non_blocking=True)
             whtmix.forward(xd, gd, out=yd)
-            yh.copy_(yd, non_blocking=True)
+            if w.backward:
+                whtmix.backward(xd, gd, dys[0], dx=dxs[0], dg=dgs[0])
+            for dst, src in d2h:
+                dst.copy_(src, non_blocking=True)
+        for _ in range(3):
+            e2e_step()
         torch.cuda.synchronize(dev)
         s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s2.record(stream)
         for _ in range(ke):
-            xd.copy_(xh, non_blocking=True)
-            gd.copy_(gh, non_blocking=True)
-            whtmix.forward(xd, gd, out=yd)
-            yh.copy_(yd, non_blocking=True)
+            e2e_step()
         e2.record(stream)
         torch.cuda.synchronize(dev)
         e2e_ms = s2.elapsed_time(e2) / ke
         e2e = {"value": tokens_per_step / (e2e_ms / 1e3), "unit": "tokens/s",
-               "h2d_bytes_per_step": xh.numel() * xh.element_size() + gh.numel() * gh.element_size(),
-               "d2h_bytes_per_step": yh.numel() * yh.element_size(), "steps": ke, "ms_per_step": e2e_ms}
+               "h2d_bytes_per_step": sum(src.numel() * src.element_size() for _, src in h2d),
+               "d2h_bytes_per_step": sum(dst.numel() * dst.element_size() for dst, _ in d2h),
+               "steps": ke, "ms_per_step": e2e_ms}
 
     if rank != 0:
         if world > 1:
@@ -324,13 +360,14 @@ def ours(args, w):
 
     cpu = None
     if not args.no_cpu_baseline:
-        t_med, times = oracle_time_plane(w, w.N, 3)
+        t_med, times = oracle_time_plane(w, w.N, 1 if w.backward else 3)
         cpu = {"value": w.B * w.N / (t_med * w.B), "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"one full [{w.N},{w.C}] plane of the workload (B={w.B} planes would take "
-                         f"{w.B * t_med:.2f} s), float64 oracle, median of 3 runs: "
+                         f"{w.B * t_med:.2f} s), float64 oracle{' forward + backward' if w.backward else ''}, "
+                         f"median of {len(times)} run(s): "
                          + ", ".join(f"{t:.2f}" for t in times) + " s"}
 
-    line = {"metric": "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s", "n_gpus": world,
+    line = {"metric": "WHTMix fwd+bwd tokens/s" if w.backward else "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
@@ -345,8 +382,9 @@ def ours(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic_from_profile(w.name),
                          "peak_kind": peak_kind, "algorithmic_bytes_per_launch": ideal,
-                         "kernel": kernel_name(w) + " (one launch per step)"},
-            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K, "clocks": clocks}
+                         "kernel": kernel_name(w) + (" + k_backward_m (two launches per step)" if w.backward
+                                                     else " (one launch per step)")},
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K * launches_per_step, "clocks": clocks}
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -362,8 +400,6 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     w = inputs.WORKLOADS[args.workload]
-    if w.backward:
-        raise SystemExit("the bench times the forward; the training-step workload is a parity case")
     if args.impl == "reference":
         reference_arm(args, w)
     else:
