@@ -390,6 +390,47 @@ def ours(args, w):
         dist.destroy_process_group()
 
 
+def sweep(args):
+    """Isolated-mixer latency against the token count N at batch 1, C = 64 (the paper's Section
+    IV-C measurement of the mixer alone, power-of-two N, no padding).  Each point: one
+    whtmix_forward call on resident bf16 inputs, CUDA events around each of 200 calls after 20
+    warm-up calls on the same buffers (a latency, so the caches are warm as in a repeated call).
+    Prints one JSON line with the per-N medians and the log-log slope."""
+    import math
+    import numpy as np
+    import torch
+    from paper_2607_25234_gb300 import whtmix
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    C = 64
+    points = []
+    for N in [1 << k for k in range(10, 17)]:
+        d = inputs.make_inputs(1, N, C, "bf16", seed=0)
+        x = torch.from_numpy(d["x"].view(np.int16)).to(dev).view(torch.bfloat16)
+        g = torch.from_numpy(d["g"]).to(dev)
+        y = torch.empty_like(x)
+        for _ in range(20):
+            whtmix.forward(x, g, out=y)
+        whtmix.sync()
+        ts = []
+        for _ in range(200):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            whtmix.forward(x, g, out=y)
+            b.record()
+            ts.append((a, b))
+        torch.cuda.synchronize(dev)
+        us = statistics.median(a.elapsed_time(b) * 1e3 for a, b in ts)
+        points.append({"N": N, "C": C, "us": us, "kernel": kernel_name(inputs.Workload("s", 1, N, C, "bf16"))})
+    xs = [math.log(p["N"]) for p in points]
+    ys = [math.log(p["us"]) for p in points]
+    mx, my = sum(xs) / len(xs), sum(ys) / len(ys)
+    slope = sum((a - mx) * (b - my) for a, b in zip(xs, ys)) / sum((a - mx) ** 2 for a in xs)
+    print(json.dumps({"metric": "WHTMix isolated mixer latency vs N (batch 1, C=64, bf16)", "unit": "us",
+                      "points": points, "loglog_slope": slope,
+                      "paper_context": "paper (RTX 4090): isolated WHTMix slope 0.25, attention 1.70"}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -398,7 +439,11 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=inputs.WORKLOAD_ORDER)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="isolated-mixer latency vs N (batch 1, C=64) instead")
     args = ap.parse_args()
+    if args.sweep:
+        sweep(args)
+        return
     w = inputs.WORKLOADS[args.workload]
     if args.impl == "reference":
         reference_arm(args, w)
