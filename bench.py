@@ -52,6 +52,15 @@ def kernel_name(w) -> str:
     return "k_forward_s" if m <= 13 else "k_forward_m"
 
 
+def backward_kernel_name(w) -> str:
+    """The kernel one whtmix_backward call launches for this workload (mirrors the C ABI's dispatch)."""
+    m = (w.N * w.C).bit_length() - 1
+    if w.dtype in ("f32", "bf16") and 14 <= m <= 21:
+        r = 14 if m == 21 else 13
+        return f"k_backward_fast<{w.dtype}, R={r}, Q={m - r}>"
+    return "k_backward_s" if m <= 13 else "k_backward_m"
+
+
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     for f in sorted(KERNEL_SOURCES):
@@ -382,7 +391,7 @@ def ours(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic_from_profile(w.name),
                          "peak_kind": peak_kind, "algorithmic_bytes_per_launch": ideal,
-                         "kernel": kernel_name(w) + (" + k_backward_m (two launches per step)" if w.backward
+                         "kernel": kernel_name(w) + (f" + {backward_kernel_name(w)} (two launches per step)" if w.backward
                                                      else " (one launch per step)")},
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K * launches_per_step, "clocks": clocks}
     print(json.dumps(line), flush=True)

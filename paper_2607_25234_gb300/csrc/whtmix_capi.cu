@@ -188,6 +188,11 @@ bool use_fast_forward(int dtype, int m) {
   return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 23;
 }
 
+// The fast backward (whtmix_fast_bwd.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^21.
+bool use_fast_backward(int dtype, int m) {
+  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 21;
+}
+
 template <int D>
 int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
   using A = typename Tr<D>::A;
@@ -205,6 +210,12 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
       return launch(k_forward_s<D>, false, sms, (P.B + ppt - 1) / ppt, tile_bytes, P, stream);
     }
     return launch(k_forward_m<D>, true, sms, static_cast<long long>(P.gp) << (m - TILE_BITS), tile_bytes, P, stream);
+  }
+  if constexpr (D != DT_I32) {
+    if (use_fast_backward(D, m)) {
+      const cudaError_t e = D == DT_BF16 ? fast::backward_bf16(P, sms, stream) : fast::backward_f32(P, sms, stream);
+      return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+    }
   }
   if (m <= TILE_BITS) {
     const long long ppt = 1ll << (TILE_BITS - m);

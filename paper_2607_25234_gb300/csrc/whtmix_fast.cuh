@@ -282,10 +282,11 @@ __device__ __forceinline__ void round_v(float2 (&a)[16][4]) {
 //     r9, ...) with lanes on (r1, r2, r9, r10, r11).  round B: r0 (inside the pairs), r3..r8,
 //     and for R = 14 r9 by one shuffle stage.
 // The row arrives through the staging area (prefetched while the previous row was processed);
-// the next row's prefetch (e0_next >= 0) is issued as soon as this row is in registers.
+// the next row's prefetch (element e0_next of src_next, if src_next is not null) is issued as
+// soon as this row is in registers.
 template <int D, int R>
 __device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, float* stg,
-                                               int wt, int worker, long long e0_next) {
+                                               int wt, int worker, const void* src_next, long long e0_next) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   float2 a[16][4];  // [vector][r1 + 2 r2]
   if constexpr (D == DT_F32) {
@@ -313,7 +314,7 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
     }
   }
   round_v(a);
-  if (e0_next >= 0) stage_row_in<D, R>(src, e0_next, stg, wt);
+  if (src_next != nullptr) stage_row_in<D, R>(src_next, e0_next, stg, wt);
   // exchange V -> P
 #pragma unroll
   for (int v = 0; v < 16; ++v)
@@ -623,7 +624,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
       const long long rn = r + RW::NWORKERS;
       row_forward_in<D, R>(P.x, (b0 << m) + (r << R), ws + (r << R), xbuf, stg, wt, worker,
-                           rn < re ? (b0 << m) + (rn << R) : -1);
+                           rn < re ? P.x : nullptr, (b0 << m) + (rn << R));
     }
     if (!grid_sync(P.bar, &flag)) break;
     // phase 2: column bits, gain, column bits

@@ -1,4 +1,4 @@
-// whtmix_fast_launch.cuh -- host-side launcher of the fast forward kernels for one I/O dtype.
+// whtmix_fast_launch.cuh -- host-side launcher of the fast forward and backward kernels for one I/O dtype.
 // Included by whtmix_fast_f32.cu and whtmix_fast_bf16.cu (one translation unit each, compiled in
 // parallel).  Returns a cudaError_t; the C ABI maps it to a status.
 #pragma once
@@ -9,6 +9,7 @@
 #include <mutex>
 
 #include "whtmix_fast.cuh"
+#include "whtmix_fast_bwd.cuh"
 
 namespace whtmix {
 namespace fast {
@@ -39,10 +40,8 @@ inline cudaError_t occupancy_cached(const void* kernel, size_t smem, int* occ) {
 // Every variant requests more than half an SM's shared memory, so exactly one CTA runs per SM:
 // two CTAs on one SM would both ask for all 512 TMEM columns, and the second would wait in
 // tcgen05.alloc while the first waits for it at the device-wide barrier.
-template <int D, int R, int Q>
-cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
+inline cudaError_t launch_persistent(const void* k, const Params& P, int sms, cudaStream_t stream) {
   const size_t smem = SMEM_BYTES;
-  const void* k = reinterpret_cast<const void*>(k_forward_fast<D, R, Q>);
   int occ = 0;
   cudaError_t e = occupancy_cached(k, smem, &occ);
   if (e != cudaSuccess) return e;
@@ -50,6 +49,14 @@ cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
   Params p = P;
   void* args[] = {&p};
   return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, smem, stream);
+}
+template <int D, int R, int Q>
+cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
+  return launch_persistent(reinterpret_cast<const void*>(k_forward_fast<D, R, Q>), P, sms, stream);
+}
+template <int D, int R, int Q>
+cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
+  return launch_persistent(reinterpret_cast<const void*>(k_backward_fast<D, R, Q>), P, sms, stream);
 }
 
 // Rows of 2^13 elements up to 2^22-element planes; rows of 2^14 for 2^23 (columns of at most
@@ -71,9 +78,28 @@ cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
   }
 }
 
+// Backward: columns of at most 128 rows (the transformed X column of a 128-row column is parked
+// in TMEM), so rows of 2^13 up to 2^20-element planes and rows of 2^14 for 2^21.
+template <int D>
+cudaError_t launch_backward(const Params& P, int sms, cudaStream_t stream) {
+  switch (P.m) {
+    case 14: return launch_bwd_one<D, 13, 1>(P, sms, stream);
+    case 15: return launch_bwd_one<D, 13, 2>(P, sms, stream);
+    case 16: return launch_bwd_one<D, 13, 3>(P, sms, stream);
+    case 17: return launch_bwd_one<D, 13, 4>(P, sms, stream);
+    case 18: return launch_bwd_one<D, 13, 5>(P, sms, stream);
+    case 19: return launch_bwd_one<D, 13, 6>(P, sms, stream);
+    case 20: return launch_bwd_one<D, 13, 7>(P, sms, stream);
+    case 21: return launch_bwd_one<D, 14, 7>(P, sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 // Entry points defined in whtmix_fast_f32.cu / whtmix_fast_bf16.cu.
 cudaError_t forward_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream);
+cudaError_t backward_f32(const Params& P, int sms, cudaStream_t stream);
+cudaError_t backward_bf16(const Params& P, int sms, cudaStream_t stream);
 
 }  // namespace fast
 }  // namespace whtmix

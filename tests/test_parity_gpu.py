@@ -136,8 +136,14 @@ def test_forward_sweep(B, N, C, dtype):
     run_forward(B, N, C, dtype, seed=B + N + C)
 
 
-@pytest.mark.parametrize("B,N,C", [(1, 1, 1), (3, 4, 2), (5, 32, 16), (2, 64, 128), (3, 128, 128),
-                                   (4, 1024, 64), (2, 8192, 2), (1, 1 << 17, 4), (6, 512, 16)])
+BWD_SWEEP = [(1, 1, 1), (3, 4, 2), (5, 32, 16), (2, 64, 128), (6, 512, 16),
+             # every column height of the fast backward, N*C = 2^(13+Q) with Q = 1..7 (rows of 2^13)
+             # and 2^21 (rows of 2^14); odd batches leave a short last plane group
+             (3, 128, 128), (2, 8192, 2), (3, 256, 128), (4, 1024, 64), (5, 2048, 64), (2, 64, 4096),
+             (1, 1 << 17, 4), (3, 1024, 1024), (3, 8192, 256), (1, 2, 1 << 20)]
+
+
+@pytest.mark.parametrize("B,N,C", BWD_SWEEP)
 @pytest.mark.parametrize("dtype", ["f32", "bf16", "i32"])
 def test_backward_sweep(B, N, C, dtype):
     run_backward(B, N, C, dtype, seed=2 * B + N + C)
