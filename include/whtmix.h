@@ -102,9 +102,9 @@ WHTMIX_API int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype
 
 /* Same as whtmix_forward / whtmix_backward with a caller-owned device workspace of at least
  * whtmix_workspace_bytes() bytes, 256-byte aligned.  Its first 256 bytes hold a device-wide
- * barrier (an arrival count, a generation word and an error word) and must be zero before the
- * first call that uses the buffer (cudaMemset); every call that completes leaves the count and
- * the error word zero (the generation word keeps advancing, which is harmless).  Calls sharing
+ * barrier (32-bit words: arrival count, generation, error, second arrival count) and must be zero
+ * before the first call that uses the buffer (cudaMemset); every call that completes leaves both
+ * counts and the error word zero (the generation word keeps advancing, which is harmless).  Calls sharing
  * a workspace must be ordered on one stream. */
 WHTMIX_API int whtmix_forward_ex(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
                       int dtype, void *workspace, size_t workspace_bytes, void *stream);

@@ -593,6 +593,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 9) || (R == 14 && Q == 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  GridSync gsync(P.bar, &flag);
   __shared__ uint32_t tmem_slot;
   constexpr bool USE_TMEM = Q >= 8;
   using RW = Row<R>;
@@ -626,12 +627,12 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
       row_forward_in<D, R>(P.x, (b0 << m) + (r << R), ws + (r << R), xbuf, stg, wt, worker,
                            rn < re ? P.x : nullptr, (b0 << m) + (rn << R));
     }
-    if (!grid_sync(P.bar, &flag)) break;
+    if (!gsync()) break;
     // phase 2: column bits, gain, column bits
     if constexpr (USE_TMEM) col_pass_tmem<Q, R>(ws, g, P.scale, m, cb, ce, tlane);
     else if constexpr (Q == 7) col_pass_single128<R>(ws, g, P.scale, m, cb, ce);
     else col_pass_pairs<Q, R>(ws, g, P.scale, m, cb, ce);
-    if (!grid_sync(P.bar, &flag)) break;
+    if (!gsync()) break;
     // phase 3: ws -> Y, row bits
     if (rb + worker < re) stage_row_out<R>(ws + ((rb + worker) << R), stg, wt);
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
@@ -639,7 +640,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
       row_forward_out<D, R>(ws + (r << R), P.y, (b0 << m) + (r << R), xbuf, stg, wt, worker,
                             rn < re ? ws + (rn << R) : nullptr);
     }
-    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) break;
+    if (b0 + P.gp < P.B && !gsync()) break;
   }
   if constexpr (USE_TMEM) {
     tmem_fence_before();

@@ -146,6 +146,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 7) || (R == 14 && Q == 7), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  GridSync gsync(P.bar, &flag);
   __shared__ uint32_t tmem_slot;
   constexpr bool USE_TMEM = Q == 7;
   using RW = Row<R>;
@@ -185,7 +186,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
                              e0_of(un));
       }
     }
-    if (!grid_sync(P.bar, &flag)) break;
+    if (!gsync()) break;
     // phase 2: columns of both, product, gain
     {
       const long long cols = nb << R;
@@ -193,7 +194,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
       const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
       col_pass_bwd<Q, R>(wsx, wsd, g, P.scale, m, cb, ce, tcol);
     }
-    if (!grid_sync(P.bar, &flag)) break;
+    if (!gsync()) break;
     // phase 3: wsd -> dX, row bits; then this CTA's dG positions
     {
       const long long rb = rows * blockIdx.x / gridDim.x, re = rows * (blockIdx.x + 1) / gridDim.x;
@@ -205,7 +206,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
       }
       dg_reduce<R>(dg, wsx, m, nb, b0 == 0, lb, le);
     }
-    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) break;
+    if (b0 + P.gp < P.B && !gsync()) break;
   }
   if constexpr (USE_TMEM) {
     tmem_fence_before();

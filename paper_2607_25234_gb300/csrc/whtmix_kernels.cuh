@@ -37,10 +37,11 @@ enum DType { DT_F32 = 0, DT_BF16 = 1, DT_I32 = 2 };
 
 // Device-wide barrier state; lives in the first 256 bytes of the workspace.
 struct GridBarrier {
-  unsigned int count;  // arrivals at the current barrier (back to 0 after each barrier)
-  unsigned int gen;    // generation, bumped by the last arrival
-  unsigned int err;    // non-zero once a wait gave up
-  unsigned int pad[61];
+  unsigned int count;      // arrivals at a barrier of even generation (back to 0 after it)
+  unsigned int gen;        // generation, bumped by the last arrival
+  unsigned int err;        // non-zero once a wait gave up
+  unsigned int count_odd;  // arrivals at a barrier of odd generation (back to 0 after it)
+  unsigned int pad[60];
 };
 static_assert(sizeof(GridBarrier) == 256, "barrier header is 256 bytes");
 
@@ -273,37 +274,52 @@ __device__ __forceinline__ unsigned int ld_acquire(const unsigned int* p) {
   return v;
 }
 
-// All CTAs of a cooperative launch call this the same number of times.  Returns false (and
-// sets bar->err) if this CTA gave up after BARRIER_TIMEOUT_NS; the caller then returns.
-__device__ __forceinline__ bool grid_sync(GridBarrier* bar, int* flag) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    const unsigned int gen = ld_acquire(&bar->gen);
-    __threadfence();
-    const unsigned int arrived = atomicAdd(&bar->count, 1u);
-    if (arrived == gridDim.x - 1) {
-      atomicExch(&bar->count, 0u);
+// Device-wide barrier of a cooperative launch; every CTA calls it the same number of times.
+// Returns false (and sets bar->err) if this CTA gave up after BARRIER_TIMEOUT_NS; the caller
+// then returns.  Thread 0 of each CTA reads the generation word once, at kernel start (it cannot
+// advance before this CTA arrives), and counts the barriers itself afterwards, so an arrival is
+// one fence and one atomic.  Barriers of even and odd generation count arrivals in separate words:
+// the last arrival releases the others first and clears its counter afterwards, off the critical
+// path, since that counter is next used two barriers later, which no CTA reaches before the last
+// arrival has passed the barrier in between.
+struct GridSync {
+  GridBarrier* bar;
+  int* flag;          // shared: thread 0's verdict for the CTA
+  unsigned int gen;   // thread 0: generation of the next barrier
+  __device__ __forceinline__ GridSync(GridBarrier* b, int* f) : bar(b), flag(f), gen(0) {
+    if (threadIdx.x == 0) gen = ld_acquire(&b->gen);
+  }
+  __device__ __forceinline__ bool operator()() {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int ok = 1;
+      unsigned int* count = (gen & 1u) ? &bar->count_odd : &bar->count;
       __threadfence();
-      atomicAdd(&bar->gen, 1u);
-    } else {
-      // Spin on the generation word (no sleep: the wait is ~1 us and a sleep quantum would add
-      // to it); the clock is read once per 256 polls to bound the wait.
-      const unsigned long long t0 = global_ns();
-      for (unsigned int polls = 1; ld_acquire(&bar->gen) == gen; ++polls) {
-        if ((polls & 255u) == 0 && global_ns() - t0 > BARRIER_TIMEOUT_NS) {
-          atomicOr(&bar->err, 1u);
-          ok = 0;
-          break;
+      const unsigned int arrived = atomicAdd(count, 1u);
+      if (arrived == gridDim.x - 1) {
+        __threadfence();
+        atomicAdd(&bar->gen, 1u);
+        atomicExch(count, 0u);
+      } else {
+        // Spin on the generation word (no sleep: the wait is ~1 us and a sleep quantum would add
+        // to it); the clock is read once per 256 polls to bound the wait.
+        const unsigned long long t0 = global_ns();
+        for (unsigned int polls = 1; ld_acquire(&bar->gen) == gen; ++polls) {
+          if ((polls & 255u) == 0 && global_ns() - t0 > BARRIER_TIMEOUT_NS) {
+            atomicOr(&bar->err, 1u);
+            ok = 0;
+            break;
+          }
         }
       }
+      __threadfence();
+      ++gen;
+      *flag = ok;
     }
-    __threadfence();
-    *flag = ok;
+    __syncthreads();
+    return *flag != 0;
   }
-  __syncthreads();
-  return *flag != 0;
-}
+};
 
 // ---------------------------------------------------------------------------------------------
 // Forward, plan S (no device-wide barrier: launched as an ordinary persistent grid).
@@ -333,6 +349,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* ws = static_cast<A*>(P.ws);
   const int m = P.m, q = m - TILE_BITS, w = TILE_BITS - q;
@@ -349,7 +366,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
       store_ws_contig(tA, ws, (b << m) + (rt << TILE_BITS));
       __syncthreads();
     }
-    if (!grid_sync(P.bar, &flag)) return;
+    if (!gsync()) return;
     // phase 2: bits [13, m) forward, gain, inverse on each column tile, ws -> ws
     for (long long u = blockIdx.x; u < units; u += gridDim.x) {
       const long long b = u >> q, col0 = (u & ((1ll << q) - 1)) << w;
@@ -359,7 +376,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
       store_ws_col(tA, ws, (b << m) + col0, w);
       __syncthreads();
     }
-    if (!grid_sync(P.bar, &flag)) return;
+    if (!gsync()) return;
     // phase 3: bits [0, 13) again, ws -> Y
     for (long long u = blockIdx.x; u < units; u += gridDim.x) {
       const long long b = u >> q, rt = u & ((1ll << q) - 1);
@@ -369,7 +386,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
       store_contig<D>(tA, P.y, ((b0 + b) << m) + (rt << TILE_BITS), TILE);
       __syncthreads();
     }
-    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) return;
+    if (b0 + P.gp < P.B && !gsync()) return;
     (void)L;
   }
 }
@@ -380,6 +397,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_s(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* tB = tA + TILE;
   A* ws = static_cast<A*>(P.ws);
@@ -401,13 +419,13 @@ __global__ void __launch_bounds__(THREADS) k_backward_s(Params P) {
       store_contig<D>(tB, P.dx, (b0 + tb) << m, n);
       __syncthreads();
     }
-    if (!grid_sync(P.bar, &flag)) return;
+    if (!gsync()) return;
     for (long long l = blockIdx.x * (long long)THREADS + threadIdx.x; l < L; l += (long long)gridDim.x * THREADS) {
       A acc = b0 == 0 ? A(0) : ld_ws(dg, l);
       for (long long b = 0; b < nb; ++b) acc = acc + ld_ws(ws, (b << m) + l);
       dg[l] = acc;
     }
-    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) return;
+    if (b0 + P.gp < P.B && !gsync()) return;
   }
 }
 
@@ -419,6 +437,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* tB = tA + TILE;
   A* tC = tB + TILE;
@@ -439,7 +458,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
       store_ws_contig(tA, is_dy ? wsd : wsx, (b << m) + (rt << TILE_BITS));
       __syncthreads();
     }
-    if (!grid_sync(P.bar, &flag)) return;
+    if (!gsync()) return;
     for (long long ct = blockIdx.x; ct < (1ll << q); ct += gridDim.x) {
       const long long col0 = ct << w;
       if (b0 == 0) {
@@ -459,7 +478,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
       store_ws_col(tC, dg, col0, w);
       __syncthreads();
     }
-    if (!grid_sync(P.bar, &flag)) return;
+    if (!gsync()) return;
     for (long long u = blockIdx.x; u < units; u += gridDim.x) {
       const long long b = u >> q, rt = u & ((1ll << q) - 1);
       load_ws_contig(tA, wsd, (b << m) + (rt << TILE_BITS));
@@ -468,7 +487,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
       store_contig<D>(tA, P.dx, ((b0 + b) << m) + (rt << TILE_BITS), TILE);
       __syncthreads();
     }
-    if (b0 + P.gp < P.B && !grid_sync(P.bar, &flag)) return;
+    if (b0 + P.gp < P.B && !gsync()) return;
   }
 }
 

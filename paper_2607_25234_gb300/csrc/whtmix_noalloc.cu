@@ -127,7 +127,7 @@ extern "C" WHTMIX_API int whtmix_forward_noalloc(const void* x, const void* gain
   if (gp > B) gp = B;
   P.gp = static_cast<int>(gp);
   if (m > TILE_BITS) {
-    // The barrier's arrival count and error word must start at zero; a call that gave up
+    // The barrier's arrival counts and error word must start at zero; a call that gave up
     // part-way could have left them set, so clear the header before every launch (a memset
     // on the stream, no allocation).  The workspace itself is fully written before it is read.
     if (cudaMemsetAsync(scratch, 0, WHTMIX_NOALLOC_HEADER_BYTES, stream) != cudaSuccess) return WHTMIX_ERR_CUDA;

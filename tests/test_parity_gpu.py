@@ -221,7 +221,7 @@ def test_ex_variant_matches_plain_call():
     torch.cuda.synchronize()
     assert torch.equal(y1, y2) and torch.equal(dx1, dx2) and torch.equal(dg1, dg2)
     header = ws[:256].view(torch.int32).cpu()
-    assert header[0].item() == 0 and header[2].item() == 0  # arrival count and error word back at zero
+    assert header[0].item() == 0 and header[2].item() == 0 and header[3].item() == 0  # counts and error word at zero
 
 
 def test_empty_batch_and_errors_on_gpu():
