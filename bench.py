@@ -48,7 +48,8 @@ def kernel_name(w) -> str:
     m = (w.N * w.C).bit_length() - 1
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 14 if m == 23 else 13
-        return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}>"
+        sep = ", separable gains" if w.gains == "separable" else ""
+        return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}>"
     return "k_forward_s" if m <= 13 else "k_forward_m"
 
 
@@ -148,11 +149,15 @@ def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
     x = inputs.as_float64(d["x"], w.dtype)
     g = d["g"].astype(np.float64)
     dy = inputs.as_float64(d["dy"], w.dtype) if w.backward else None
+    g_t, g_c = (a.astype(np.float64) for a in inputs.make_log_gains(n_tokens, w.C, 0))
     oracle.forward(x[:, :8, :], g[:8, :])  # load / compile outside the timing
     times = []
     for _ in range(reps):
         t = time.perf_counter()
-        oracle.forward(x, g)
+        if w.gains == "separable":
+            oracle.forward_separable(x, g_t, g_c)
+        else:
+            oracle.forward(x, g)
         if dy is not None:
             oracle.backward(x, g, dy)
         times.append(time.perf_counter() - t)
@@ -176,11 +181,16 @@ def reference_arm(args, w):
     d = inputs.make_inputs(1, n, w.C, w.dtype, seed=0, n_valid=None if w.n_valid is None else min(w.n_valid, n))
     x = inputs.as_float64(d["x"], w.dtype)
     g = d["g"].astype(np.float64)
+    if w.gains == "separable":
+        g_t, g_c = (a.astype(np.float64) for a in inputs.make_log_gains(n, w.C, 0))
+        run = lambda: oracle.forward_separable(x, g_t, g_c)
+    else:
+        run = lambda: oracle.forward(x, g)
     for _ in range(args.warmup):
-        oracle.forward(x, g)
+        run()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle.forward(x, g)
+        run()
     el = time.perf_counter() - t0
     value = args.steps * n / el
     sample = f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s)"
@@ -230,7 +240,9 @@ def ours(args, w):
     x_host = torch.from_numpy(d["x"].view(np.int16) if w.dtype == "bf16" else d["x"])
     if w.dtype == "bf16":
         x_host = x_host.view(torch.bfloat16)
-    g_host = torch.from_numpy(d["g"])
+    # the gains: G [N, C], or for the separable workload g_t [N] and g_c [C] in one buffer
+    sep = w.gains == "separable"
+    g_host = torch.from_numpy(np.concatenate([d["g_t"], d["g_c"]]) if sep else d["g"])
     x0 = x_host.to(dev)
     g0 = g_host.to(dev)
     # a training step (forward + backward) also reads dY and writes dX and dG
@@ -257,11 +269,15 @@ def ours(args, w):
     bargs_c = [(dys[i].data_ptr(), dxs[i].data_ptr(), dgs[i].data_ptr()) for i in range(nsets)] if w.backward else None
     fwd = lib.whtmix_forward
     bwd = lib.whtmix_backward
+    fwd_sep = lib.whtmix_forward_separable
     launches_per_step = 2 if w.backward else 1
 
     def step(i):
         a = args_c[i % nsets]
-        rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
+        if sep:
+            rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, w.N, w.C, code, sp)
+        else:
+            rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
         if rc != 0:
             raise whtmix.WhtmixError(rc, "whtmix_forward")
         if w.backward:
@@ -342,7 +358,10 @@ def ours(args, w):
         def e2e_step():
             for dst, src in h2d:
                 dst.copy_(src, non_blocking=True)
-            whtmix.forward(xd, gd, out=yd)
+            if sep:
+                whtmix.forward_separable(xd, gd[:w.N], gd[w.N:], out=yd)
+            else:
+                whtmix.forward(xd, gd, out=yd)
             if w.backward:
                 whtmix.backward(xd, gd, dys[0], dx=dxs[0], dg=dgs[0])
             for dst, src in d2h:
@@ -380,7 +399,7 @@ def ours(args, w):
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
-                       "f32" if w.dtype != "i32" else "i32", "parallelism": f"replicas{world}",
+                       "f32" if w.dtype != "i32" else "i32", "gains": w.gains, "parallelism": f"replicas{world}",
                        "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / 2**20:.0f} MiB, "
                              f"{nsets * set_bytes / l2:.1f}x L2)"},
             "hbm_gbs": achieved, "pct_of_measured_peak": 100.0 * achieved / peak,

@@ -137,3 +137,23 @@ def backward(x: np.ndarray, g: np.ndarray, dy: np.ndarray):
     dg = np.empty((N, C), dtype=np.float64)
     _check(lib.oracle_backward_f64(_ptr(xx), _ptr(gg), _ptr(dd), _ptr(dx), _ptr(dg), B, N, C))
     return dx.reshape(x.shape), dg
+
+
+def separable_gains(g_t: np.ndarray, g_c: np.ndarray) -> np.ndarray:
+    """G[n, c] = exp(g_t[n]) exp(g_c[c]) in float64: the per-frequency log gains of the token mix
+    (Eq. 3) and of the channel mix (Eq. 2), Section III-B, combined into the one 2D gain plane they
+    amount to (the two mixes act on different axes)."""
+    return np.outer(np.exp(np.asarray(g_t, dtype=np.float64)), np.exp(np.asarray(g_c, dtype=np.float64)))
+
+
+def forward_separable(x: np.ndarray, g_t: np.ndarray, g_c: np.ndarray) -> np.ndarray:
+    """WHTMix forward with the log-domain gains (float64)."""
+    return forward(np.asarray(x, dtype=np.float64), separable_gains(g_t, g_c))
+
+
+def backward_separable(x: np.ndarray, g_t: np.ndarray, g_c: np.ndarray, dy: np.ndarray):
+    """(dX, dg_t, dg_c) of forward_separable: dX as in backward(); by the chain rule through
+    G = exp(g_t) exp(g_c)^T, dg_t[n] = sum_c dG[n, c] G[n, c] and dg_c[c] = sum_n dG[n, c] G[n, c]."""
+    G = separable_gains(g_t, g_c)
+    dx, dG = backward(np.asarray(x, dtype=np.float64), G, np.asarray(dy, dtype=np.float64))
+    return dx, (dG * G).sum(axis=1), (dG * G).sum(axis=0)

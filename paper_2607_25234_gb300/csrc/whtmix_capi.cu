@@ -298,6 +298,183 @@ int run(bool backward, const void* x, const void* g, const void* dy, void* y_or_
   }
 }
 
+// ---- separable log gains (Section III-B, Eq. 2-3): G[n, c] = exp(g_t[n]) exp(g_c[c]) ----
+
+constexpr int SEP_THREADS = 256;
+
+size_t align256(size_t v) { return (v + 255) & ~size_t{255}; }
+
+// G[e] = exp(g_t[e >> cbits]) * exp(g_c[e mod C]) over one plane: the same two expf values and
+// the same single rounding of their product as the separable fast forward's tables.
+__global__ void k_sep_gains(float* G, const float* gt, const float* gc, int m, int cbits) {
+  const long long L = 1ll << m, cm = (1ll << cbits) - 1;
+  for (long long e = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; e < L;
+       e += static_cast<long long>(gridDim.x) * blockDim.x)
+    G[e] = expf(gt[e >> cbits]) * expf(gc[e & cm]);
+}
+
+// dg_t[n] = sum over c of dG[n, c] G[n, c] (the chain rule through G = exp(g_t) exp(g_c)): one warp
+// per token, each lane over channels lane, lane + 32, ... in order, then a fixed shuffle tree.
+// These sums run over up to 2^30 products with cancellation, so they accumulate in float64 (the
+// products of two floats are exact there) and round once; they are outside the mixer's hot path.
+__global__ void k_sep_reduce_t(float* dgt, const float* dG, const float* G, int m, int cbits) {
+  const long long N = 1ll << (m - cbits);
+  const int C = 1 << cbits, lane = threadIdx.x & 31;
+  const long long warps = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  for (long long n = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; n < N; n += warps) {
+    double acc = 0.0;
+    for (int c = lane; c < C; c += 32)
+      acc += static_cast<double>(dG[(n << cbits) + c]) * static_cast<double>(G[(n << cbits) + c]);
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) dgt[n] = static_cast<float>(acc);
+  }
+}
+
+// dg_c[c] = sum over n of dG[n, c] G[n, c], in two fixed-order steps (float64 as above):
+// part[k][c] over the tokens of chunk k in ascending n, then the chunks in ascending k.
+__global__ void k_sep_reduce_c_part(double* part, const float* dG, const float* G, int m, int cbits,
+                                    long long rows_per_chunk, long long nchunks) {
+  const long long N = 1ll << (m - cbits);
+  const int C = 1 << cbits;
+  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < (nchunks << cbits);
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long k = i >> cbits, c = i & (C - 1);
+    const long long n0 = k * rows_per_chunk, n1 = min(N, n0 + rows_per_chunk);
+    double acc = 0.0;
+    for (long long n = n0; n < n1; ++n)
+      acc += static_cast<double>(dG[(n << cbits) + c]) * static_cast<double>(G[(n << cbits) + c]);
+    part[i] = acc;
+  }
+}
+__global__ void k_sep_reduce_c_final(float* dgc, const double* part, int cbits, long long nchunks) {
+  const long long C = 1ll << cbits;
+  for (long long c = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; c < C;
+       c += static_cast<long long>(gridDim.x) * blockDim.x) {
+    double acc = 0.0;
+    for (long long k = 0; k < nchunks; ++k) acc += part[(k << cbits) + c];
+    dgc[c] = static_cast<float>(acc);
+  }
+}
+
+unsigned grid_for(long long work, int sms) {
+  const long long blocks = (work + SEP_THREADS - 1) / SEP_THREADS;
+  const long long cap = 8ll * sms;
+  return static_cast<unsigned>(blocks < 1 ? 1 : blocks > cap ? cap : blocks);
+}
+
+// Token chunks of the dg_c reduction: enough (chunk, channel) pairs to fill the GPU.
+long long sep_chunks(int m, int cbits) {
+  const long long N = 1ll << (m - cbits);
+  long long k = (1ll << 16) >> cbits;
+  if (k < 1) k = 1;
+  return k < N ? k : N;
+}
+
+bool use_fast_separable(int dtype, int m, int cbits) {
+  return use_fast_forward(dtype, m) && cbits >= 1 && cbits <= fast::forward_row_bits(m);
+}
+
+size_t separable_workspace_bytes(int64_t B, int m, int cbits, int dtype, bool backward) {
+  const size_t base = align256(workspace_bytes(B, m, backward));
+  const size_t L = size_t{1} << m;
+  if (!backward) {
+    if (use_fast_separable(dtype, m, cbits)) return base + align256(((L >> cbits) + (size_t{1} << cbits)) * 4);
+    return base + align256(L * 4);
+  }
+  return base + 2 * align256(L * 4) + align256(static_cast<size_t>(sep_chunks(m, cbits) << cbits) * 8);
+}
+
+int run_separable(bool backward, const void* x, const float* gt, const float* gc, const void* dy, void* y_or_dx,
+                  float* dgt, float* dgc, int64_t B, int64_t N, int64_t C, int dtype, void* stream_v) {
+  int m = 0;
+  int rc = check_shape(B, N, C, dtype, &m);
+  if (rc != WHTMIX_OK) return rc;
+  if (dtype == WHTMIX_I32) return WHTMIX_ERR_BAD_DTYPE;  // log-domain gains are real
+  const int cbits = ilog2_pow2(C);
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  auto aligned4 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; };
+  const size_t N_bytes = static_cast<size_t>(N) * 4, C_bytes = static_cast<size_t>(C) * 4;
+  if (B == 0) {
+    // Empty batch: the forward has nothing to do; the backward's gradients are sums over no planes.
+    if (!backward) return WHTMIX_OK;
+    if (!dgt || !dgc) return WHTMIX_ERR_INVALID_ARG;
+    if (!aligned4(dgt) || !aligned4(dgc)) return WHTMIX_ERR_MISALIGNED;
+    if (overlap(dgt, N_bytes, dgc, C_bytes)) return WHTMIX_ERR_ALIAS;
+    int dev = 0, sms = 0;
+    rc = device_check(&dev, &sms);
+    if (rc != WHTMIX_OK) return rc;
+    cudaError_t e = cudaMemsetAsync(dgt, 0, N_bytes, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dgc, 0, C_bytes, stream);
+    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+  }
+  if (!x || !gt || !gc || !y_or_dx || (backward && (!dy || !dgt || !dgc))) return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(y_or_dx) || (backward && !aligned16(dy))) return WHTMIX_ERR_MISALIGNED;
+  if (!aligned4(gt) || !aligned4(gc) || (backward && (!aligned4(dgt) || !aligned4(dgc)))) return WHTMIX_ERR_MISALIGNED;
+  const size_t L = size_t{1} << m;
+  const size_t plane_bytes = static_cast<size_t>(B) * L * elem_size(dtype);
+  void* out = y_or_dx;
+  const void* in = backward ? dy : x;
+  if (out != in && overlap(out, plane_bytes, in, plane_bytes)) return WHTMIX_ERR_ALIAS;
+  if (overlap(out, plane_bytes, gt, N_bytes) || overlap(out, plane_bytes, gc, C_bytes)) return WHTMIX_ERR_ALIAS;
+  if (backward) {
+    if (overlap(out, plane_bytes, x, plane_bytes)) return WHTMIX_ERR_ALIAS;
+    const void* ins[5] = {x, dy, gt, gc, out};
+    const size_t ins_bytes[5] = {plane_bytes, plane_bytes, N_bytes, C_bytes, plane_bytes};
+    for (int i = 0; i < 5; ++i)
+      if (overlap(dgt, N_bytes, ins[i], ins_bytes[i]) || overlap(dgc, C_bytes, ins[i], ins_bytes[i]))
+        return WHTMIX_ERR_ALIAS;
+    if (overlap(dgt, N_bytes, dgc, C_bytes)) return WHTMIX_ERR_ALIAS;
+  }
+  int dev = 0, sms = 0;
+  rc = device_check(&dev, &sms);
+  if (rc != WHTMIX_OK) return rc;
+  void* ws = nullptr;
+  rc = cached_workspace(dev, stream, separable_workspace_bytes(B, m, cbits, dtype, backward), &ws);
+  if (rc != WHTMIX_OK) return rc;
+  char* extra = static_cast<char*>(ws) + align256(workspace_bytes(B, m, backward));
+  Params P{};
+  P.x = x;
+  P.dy = dy;
+  P.bar = static_cast<GridBarrier*>(ws);
+  P.ws = static_cast<char*>(ws) + HEADER_BYTES;
+  P.B = B;
+  P.m = m;
+  P.gp = planes_per_group(B, m, backward);
+  P.scale = 1.0f / static_cast<float>(L);
+  P.gt = gt;
+  P.gc = gc;
+  P.cbits = cbits;
+  if (!backward && use_fast_separable(dtype, m, cbits)) {
+    // the gain tables go right after the plane group, where the kernel expects them
+    P.y = y_or_dx;
+    const cudaError_t e = dtype == WHTMIX_BF16 ? fast::forward_sep_bf16(P, sms, stream) : fast::forward_sep_f32(P, sms, stream);
+    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+  }
+  // Otherwise G is built in the workspace and the full-gain kernels run on it.
+  float* G = reinterpret_cast<float*>(extra);
+  k_sep_gains<<<grid_for(static_cast<long long>(L), sms), SEP_THREADS, 0, stream>>>(G, gt, gc, m, cbits);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e);
+  P.g = G;
+  if (!backward) {
+    P.y = y_or_dx;
+    return dtype == WHTMIX_BF16 ? dispatch<DT_BF16>(false, P, sms, stream) : dispatch<DT_F32>(false, P, sms, stream);
+  }
+  float* dG = reinterpret_cast<float*>(extra + align256(L * 4));
+  double* part = reinterpret_cast<double*>(extra + 2 * align256(L * 4));
+  P.dx = y_or_dx;
+  P.dg = dG;
+  rc = dtype == WHTMIX_BF16 ? dispatch<DT_BF16>(true, P, sms, stream) : dispatch<DT_F32>(true, P, sms, stream);
+  if (rc != WHTMIX_OK) return rc;
+  const long long nchunks = sep_chunks(m, cbits), Nn = 1ll << (m - cbits);
+  k_sep_reduce_t<<<grid_for(Nn * 32, sms), SEP_THREADS, 0, stream>>>(dgt, dG, G, m, cbits);
+  k_sep_reduce_c_part<<<grid_for(nchunks << cbits, sms), SEP_THREADS, 0, stream>>>(part, dG, G, m, cbits,
+                                                                                    (Nn + nchunks - 1) / nchunks, nchunks);
+  k_sep_reduce_c_final<<<grid_for(1ll << cbits, sms), SEP_THREADS, 0, stream>>>(dgc, part, cbits, nchunks);
+  e = cudaGetLastError();
+  return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+}
+
 }  // namespace
 
 extern "C" {
@@ -319,6 +496,16 @@ int whtmix_forward_ex(const void* x, const void* gains, void* y, int64_t B, int6
 int whtmix_backward_ex(const void* x, const void* gains, const void* dy, void* dx, void* dgains, int64_t B, int64_t N,
                        int64_t C, int dtype, void* workspace, size_t workspace_bytes_, void* stream) {
   return run(true, x, gains, dy, dx, dgains, B, N, C, dtype, workspace, workspace_bytes_, true, stream);
+}
+
+int whtmix_forward_separable(const void* x, const float* g_t, const float* g_c, void* y, int64_t B, int64_t N,
+                             int64_t C, int dtype, void* stream) {
+  return run_separable(false, x, g_t, g_c, nullptr, y, nullptr, nullptr, B, N, C, dtype, stream);
+}
+
+int whtmix_backward_separable(const void* x, const float* g_t, const float* g_c, const void* dy, void* dx,
+                              float* dg_t, float* dg_c, int64_t B, int64_t N, int64_t C, int dtype, void* stream) {
+  return run_separable(true, x, g_t, g_c, dy, dx, dg_t, dg_c, B, N, C, dtype, stream);
 }
 
 int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype, int backward, size_t* out_bytes) {

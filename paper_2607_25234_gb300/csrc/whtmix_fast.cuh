@@ -24,6 +24,8 @@
 //   * column ranges are balanced and aligned to 8 columns (32-byte sectors).
 #pragma once
 
+#include <type_traits>
+
 #include "whtmix_kernels.cuh"
 
 namespace whtmix {
@@ -223,6 +225,17 @@ __device__ __forceinline__ void cp_async4(float* smem_dst, const float* gsrc) {
   const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gsrc) : "memory");
 }
+// Bulk prefetch into L2 of piece i of n of this CTA's 1/gridDim.x share of a buffer (16-byte
+// chunks).
+__device__ __forceinline__ void l2_prefetch_piece(const void* base, long long bytes, long long i, long long n) {
+  const long long chunks = bytes >> 4;
+  const long long s0 = chunks * blockIdx.x / gridDim.x, s1 = chunks * (blockIdx.x + 1) / gridDim.x;
+  const long long c0 = s0 + (s1 - s0) * i / n, c1 = s0 + (s1 - s0) * (i + 1) / n;
+  if (c1 > c0)
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(base) + (c0 << 4)),
+                 "r"(static_cast<unsigned>((c1 - c0) << 4))
+                 : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
@@ -379,10 +392,64 @@ __device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, 
 }
 
 // ---------------------------------------------------------------------------------------------
+// Gains as phase 2 reads them, per column: storage position sp of a workspace row, whose element
+// j is logical plane element (j << R) + sigma_inv(sp).  at() is one element of the column, at2()
+// the elements of the storage positions sp and sp + 1 (sp even), which sigma_inv keeps adjacent.
+template <int R>
+struct FullGain {  // G [N, C] as given
+  static constexpr bool SEPARABLE = false;
+  const float* g;
+  struct Col {
+    const float* p;
+  };
+  __device__ __forceinline__ Col col(int sp) const { return {g + sigma_inv(sp)}; }
+  __device__ __forceinline__ float at(const Col& c, long long j) const { return __ldg(c.p + (j << R)); }
+  __device__ __forceinline__ float2 at2(const Col& c, long long j) const {
+    return __ldg(reinterpret_cast<const float2*>(c.p + (j << R)));
+  }
+};
+// Separable log gains (Section III-B, Eq. 2-3): G[n, c] = exp(g_t[n]) exp(g_c[c]), from two tables
+// phase 1 builds in the workspace.  With C = 2^cb, 1 <= cb <= R, a column holds one channel
+// c = s mod C (s = sigma_inv(sp)) and the tokens n = (j << (R - cb)) + (s >> cb), so the token
+// table is stored column-major, etT[(n mod 2^(R-cb)) * 2^Q + (n >> (R-cb))] = exp(g_t[n]): a column's
+// gains are then consecutive floats (compile-time offsets from one pointer), and ec[c] = exp(g_c[c]).
+// at2's second position is channel c + 1 of the same token.  The tables are written during the
+// launch, before the barrier that opens phase 2, so they are read with ordinary (coherent) loads.
+template <int R, int Q>
+struct SepGain {
+  static constexpr bool SEPARABLE = true;
+  const float* etT;
+  const float* ec;
+  int cb;
+  struct Col {
+    const float* p;
+    float e0, e1;
+  };
+  __device__ __forceinline__ Col col(int sp) const {
+    const int s = sigma_inv(sp), c = s & ((1 << cb) - 1);
+    return {etT + (static_cast<long long>(s >> cb) << Q), ec[c], ec[c | 1]};
+  }
+  __device__ __forceinline__ float at(const Col& c, long long j) const { return c.p[j] * c.e0; }
+  __device__ __forceinline__ float2 at2(const Col& c, long long j) const {
+    const float t = c.p[j];
+    return make_float2(t * c.e0, t * c.e1);
+  }
+  // rows j and j + 1 (j even: one 8-byte load)
+  __device__ __forceinline__ float2 rows2(const Col& c, long long j) const {
+    return mul2(*reinterpret_cast<const float2*>(c.p + j), make_float2(c.e0, c.e0));
+  }
+};
+// Entry i of the column-major token table built by phase 1: exp(g_t[n]) for the token n it holds.
+template <int R, int Q>
+__device__ __forceinline__ long long sep_token_of(long long i, int cb) {
+  return ((i & ((1ll << Q) - 1)) << (R - cb)) | (i >> Q);
+}
+
+// ---------------------------------------------------------------------------------------------
 // Phase 2, register variant (Q <= 6): a thread owns two adjacent storage positions (one logical
 // column pair) x 2^Q rows.
-template <int Q, int R>
-__device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
+template <int Q, int R, class GainT>
+__device__ __forceinline__ void col_pass_pairs(float* ws, const GainT& gain, float scale, int m, long long u_begin, long long u_end) {
   constexpr int NR = 1 << Q;
   const float2 sc = make_float2(scale, scale);
   for (long long u0 = u_begin; u0 < u_end; u0 += 2 * THREADS) {
@@ -391,13 +458,13 @@ __device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float 
     const long long b = u >> R;
     const int sp = static_cast<int>(u & ((1 << R) - 1));  // storage position (even); sp + 1 is column c + 1
     float* base = ws + (b << m) + sp;
-    const float* gb = g + sigma_inv(sp);
+    const auto gc = gain.col(sp);
     float2 v[NR];
 #pragma unroll
     for (int j = 0; j < NR; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << R)));
     bfly_all<NR>(v);
 #pragma unroll
-    for (int j = 0; j < NR; ++j) v[j] = mul2(v[j], mul2(__ldg(reinterpret_cast<const float2*>(gb + (static_cast<long long>(j) << R))), sc));
+    for (int j = 0; j < NR; ++j) v[j] = mul2(v[j], mul2(gain.at2(gc, j), sc));
     bfly_all<NR>(v);
 #pragma unroll
     for (int j = 0; j < NR; ++j) __stcg(reinterpret_cast<float2*>(base + (static_cast<long long>(j) << R)), v[j]);
@@ -405,15 +472,15 @@ __device__ __forceinline__ void col_pass_pairs(float* ws, const float* g, float 
 }
 
 // Phase 2, register variant for Q = 7: a thread owns one column of 128 rows as 64 pairs (j, j + 64).
-template <int R>
-__device__ __forceinline__ void col_pass_single128(float* ws, const float* g, float scale, int m, long long u_begin, long long u_end) {
+template <int R, class GainT>
+__device__ __forceinline__ void col_pass_single128(float* ws, const GainT& gain, float scale, int m, long long u_begin, long long u_end) {
   for (long long u0 = u_begin; u0 < u_end; u0 += THREADS) {
     const long long u = u0 + threadIdx.x;
     if (u >= u_end) break;
     const long long b = u >> R;
     const int sp = static_cast<int>(u & ((1 << R) - 1));
     float* base = ws + (b << m) + sp;
-    const float* gb = g + sigma_inv(sp);
+    const auto gc = gain.col(sp);
     float2 v[64];
 #pragma unroll
     for (int j = 0; j < 64; ++j)
@@ -423,7 +490,9 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const float* g, fl
     for (int j = 0; j < 64; ++j) bf_in(v[j]);
 #pragma unroll
     for (int j = 0; j < 64; ++j) {
-      const float2 gg = make_float2(__ldg(gb + (static_cast<long long>(j) << R)), __ldg(gb + (static_cast<long long>(j + 64) << R)));
+      float2 gg;
+      if constexpr (GainT::SEPARABLE) gg = make_float2(gain.at(gc, j), gain.at(gc, j + 64));
+      else gg = make_float2(__ldg(gc.p + (static_cast<long long>(j) << R)), __ldg(gc.p + (static_cast<long long>(j + 64) << R)));
       v[j] = mul2(v[j], mul2(gg, make_float2(scale, scale)));
     }
 #pragma unroll
@@ -452,8 +521,8 @@ __device__ __forceinline__ void pair_sync(int quarter) {
 //   round A: own ET elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
 //   round B: bits k6..k(et) forward, gain, back; each warp half takes k5 = hw
 //   round C: own ET elements, bits k0..k5 again, TMEM -> global
-template <int Q, int R>
-__device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float scale, int m, long long u_begin,
+template <int Q, int R, class GainT>
+__device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, float scale, int m, long long u_begin,
                                               long long u_end, uint32_t tlane) {
   constexpr int ET_BITS = Q - 1;                       // 8, 7 for Q = 9, 8
   constexpr int ET = 1 << ET_BITS;
@@ -473,7 +542,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
     const long long b = uu >> R;
     const int sp = static_cast<int>(uu & ((1 << R) - 1));  // storage position of the column
     float* colp = ws + (b << m) + sp;
-    const float* gcol = g + sigma_inv(sp);
+    const auto gcol = gain.col(sp);
     float* own = colp + (static_cast<long long>(hw * ET) << R);
     // round A
 #pragma unroll 1
@@ -529,7 +598,10 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 #pragma unroll
         for (int w = 0; w < W; ++w) {
           const long long j = j0 + 2 * w;
-          const float2 gg = make_float2(__ldg(gcol + (j << R)), __ldg(gcol + ((j + 1) << R)));
+          float2 gg;
+          // (the full gain's loads are written out here: through at() the compiler spills in this loop)
+          if constexpr (GainT::SEPARABLE) gg = gain.rows2(gcol, j);
+          else gg = make_float2(__ldg(gcol.p + (j << R)), __ldg(gcol.p + ((j + 1) << R)));
           v[s][w] = mul2(v[s][w], mul2(gg, sc));
         }
       }
@@ -588,7 +660,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const float* g, float s
 // ---------------------------------------------------------------------------------------------
 // Forward kernel: persistent cooperative grid (one CTA per SM), plane groups of P.gp planes,
 // three phases.  R and Q are template parameters so that every register array has a static size.
-template <int D, int R, int Q>
+template <int D, int R, int Q, bool SEP>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 9) || (R == 14 && Q == 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -620,18 +692,40 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     const long long cols = nb << R;
     const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
     const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
-    // phase 1: X -> ws, row bits
+    // phase 1: X -> ws, row bits (and, once, the separable gain tables exp(g_t), exp(g_c))
+    if constexpr (SEP) {
+      if (b0 == 0) {
+        float* tab = ws + (static_cast<long long>(P.gp) << m);
+        const long long n_t = 1ll << (m - P.cbits), n_tab = n_t + (1ll << P.cbits);
+        for (long long i = static_cast<long long>(blockIdx.x) * THREADS + threadIdx.x; i < n_tab;
+             i += static_cast<long long>(gridDim.x) * THREADS)
+          tab[i] = expf(i < n_t ? P.gt[sep_token_of<R, Q>(i, P.cbits)] : P.gc[i - n_t]);
+      }
+    }
     if (rb + worker < re) stage_row_in<D, R>(P.x, (b0 << m) + ((rb + worker) << R), stg, wt);
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
       const long long rn = r + RW::NWORKERS;
+      // G is first read in phase 2; its fetch into L2 is spread over phase 1 (one bulk prefetch
+      // per row, together the CTA's share of G), where HBM carries only X.
+      if (!SEP && b0 == 0 && wt == 0) l2_prefetch_piece(g, 4ll << m, r - rb, re - rb);
       row_forward_in<D, R>(P.x, (b0 << m) + (r << R), ws + (r << R), xbuf, stg, wt, worker,
                            rn < re ? P.x : nullptr, (b0 << m) + (rn << R));
     }
     if (!gsync()) break;
     // phase 2: column bits, gain, column bits
-    if constexpr (USE_TMEM) col_pass_tmem<Q, R>(ws, g, P.scale, m, cb, ce, tlane);
-    else if constexpr (Q == 7) col_pass_single128<R>(ws, g, P.scale, m, cb, ce);
-    else col_pass_pairs<Q, R>(ws, g, P.scale, m, cb, ce);
+    {
+      using GainT = typename std::conditional<SEP, SepGain<R, Q>, FullGain<R>>::type;
+      GainT gain;
+      if constexpr (SEP) {
+        const float* tab = ws + (static_cast<long long>(P.gp) << m);
+        gain = GainT{tab, tab + (1ll << (m - P.cbits)), P.cbits};
+      } else {
+        gain = GainT{g};
+      }
+      if constexpr (USE_TMEM) col_pass_tmem<Q, R>(ws, gain, P.scale, m, cb, ce, tlane);
+      else if constexpr (Q == 7) col_pass_single128<R>(ws, gain, P.scale, m, cb, ce);
+      else col_pass_pairs<Q, R>(ws, gain, P.scale, m, cb, ce);
+    }
     if (!gsync()) break;
     // phase 3: ws -> Y, row bits
     if (rb + worker < re) stage_row_out<R>(ws + ((rb + worker) << R), stg, wt);

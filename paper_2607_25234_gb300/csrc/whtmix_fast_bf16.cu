@@ -3,7 +3,7 @@
 
 namespace whtmix {
 namespace fast {
-cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream) { return launch_forward<DT_BF16>(P, sms, stream); }
+cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream) { return launch_forward<DT_BF16, false>(P, sms, stream); }
 cudaError_t backward_bf16(const Params& P, int sms, cudaStream_t stream) { return launch_backward<DT_BF16>(P, sms, stream); }
 }  // namespace fast
 }  // namespace whtmix

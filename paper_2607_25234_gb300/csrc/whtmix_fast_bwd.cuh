@@ -181,6 +181,8 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
       if (ub + worker < ue) stage_row_in<D, R>(src_of(ub + worker), e0_of(ub + worker), stg, wt);
       for (long long u = ub + worker; u < ue; u += RW::NWORKERS) {
         const long long un = u + RW::NWORKERS;
+        // G is first read in phase 2: its fetch into L2 is spread over the first group's rows
+        if (b0 == 0 && wt == 0) l2_prefetch_piece(g, 4ll << m, u - ub, ue - ub);
         float* dst = u < rows ? wsx + (u << R) : wsd + ((u - rows) << R);
         row_forward_in<D, R>(src_of(u), e0_of(u), dst, xbuf, stg, wt, worker, un < ue ? src_of(un) : nullptr,
                              e0_of(un));

@@ -50,9 +50,9 @@ inline cudaError_t launch_persistent(const void* k, const Params& P, int sms, cu
   void* args[] = {&p};
   return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, smem, stream);
 }
-template <int D, int R, int Q>
+template <int D, int R, int Q, bool SEP>
 cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
-  return launch_persistent(reinterpret_cast<const void*>(k_forward_fast<D, R, Q>), P, sms, stream);
+  return launch_persistent(reinterpret_cast<const void*>(k_forward_fast<D, R, Q, SEP>), P, sms, stream);
 }
 template <int D, int R, int Q>
 cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
@@ -61,22 +61,25 @@ cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
 
 // Rows of 2^13 elements up to 2^22-element planes; rows of 2^14 for 2^23 (columns of at most
 // 512 rows).  Measured on the 2^22 planes, 2^13 rows with 512-row columns beat 2^14 rows.
-template <int D>
+// SEP: separable log gains (P.gt, P.gc) instead of G; needs 1 <= P.cbits <= row bits.
+template <int D, bool SEP>
 cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
   switch (P.m) {
-    case 14: return launch_one<D, 13, 1>(P, sms, stream);
-    case 15: return launch_one<D, 13, 2>(P, sms, stream);
-    case 16: return launch_one<D, 13, 3>(P, sms, stream);
-    case 17: return launch_one<D, 13, 4>(P, sms, stream);
-    case 18: return launch_one<D, 13, 5>(P, sms, stream);
-    case 19: return launch_one<D, 13, 6>(P, sms, stream);
-    case 20: return launch_one<D, 13, 7>(P, sms, stream);
-    case 21: return launch_one<D, 13, 8>(P, sms, stream);
-    case 22: return launch_one<D, 13, 9>(P, sms, stream);
-    case 23: return launch_one<D, 14, 9>(P, sms, stream);
+    case 14: return launch_one<D, 13, 1, SEP>(P, sms, stream);
+    case 15: return launch_one<D, 13, 2, SEP>(P, sms, stream);
+    case 16: return launch_one<D, 13, 3, SEP>(P, sms, stream);
+    case 17: return launch_one<D, 13, 4, SEP>(P, sms, stream);
+    case 18: return launch_one<D, 13, 5, SEP>(P, sms, stream);
+    case 19: return launch_one<D, 13, 6, SEP>(P, sms, stream);
+    case 20: return launch_one<D, 13, 7, SEP>(P, sms, stream);
+    case 21: return launch_one<D, 13, 8, SEP>(P, sms, stream);
+    case 22: return launch_one<D, 13, 9, SEP>(P, sms, stream);
+    case 23: return launch_one<D, 14, 9, SEP>(P, sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }
+// Row bits of the fast forward for a 2^m-element plane.
+inline int forward_row_bits(int m) { return m == 23 ? 14 : 13; }
 
 // Backward: columns of at most 128 rows (the transformed X column of a 128-row column is parked
 // in TMEM), so rows of 2^13 up to 2^20-element planes and rows of 2^14 for 2^21.
@@ -100,6 +103,9 @@ cudaError_t forward_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream);
 cudaError_t backward_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t backward_bf16(const Params& P, int sms, cudaStream_t stream);
+// whtmix_fast_sep_f32.cu / whtmix_fast_sep_bf16.cu
+cudaError_t forward_sep_f32(const Params& P, int sms, cudaStream_t stream);
+cudaError_t forward_sep_bf16(const Params& P, int sms, cudaStream_t stream);
 
 }  // namespace fast
 }  // namespace whtmix

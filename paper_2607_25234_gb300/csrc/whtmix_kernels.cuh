@@ -58,6 +58,10 @@ struct Params {
   int m;             // log2(N C)
   int gp;            // planes per group
   float scale;       // 1 / (N C) for the floating-point dtypes
+  // separable log gains (fast forward only): g_t [N], g_c [C], C = 2^cbits; g is unused then
+  const float* gt;
+  const float* gc;
+  int cbits;
 };
 
 // ---- dtype traits: storage <-> accumulator (fp32 for F32/BF16, uint32 for I32) ----

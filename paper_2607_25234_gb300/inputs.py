@@ -5,7 +5,8 @@ no part of the mixer's arithmetic: it draws numbers and quantises them to the st
 
 Generator: SplitMix64 (Steele, Lea & Flood, "Fast splittable pseudorandom number generators",
 OOPSLA 2014) -> 53-bit uniforms in [0, 1) -> Box-Muller normals in float64.  Each tensor has its
-own stream: X uses ``seed``, G uses ``seed + 1`` and dY uses ``seed + 2``.
+own stream: X uses ``seed``, G uses ``seed + 1`` and dY uses ``seed + 2``; the separable log
+gains g_t and g_c use ``seed + 3`` and ``seed + 4``.
 
 Stand-in data.  The paper trains and times the mixer on joint left+right stereo token sequences
 (Section III-A; N = 2 (H/8)(W/8), C = 64) and on LRA byte sequences (Section IV-D).  None of those
@@ -90,6 +91,7 @@ class Workload:
     backward: bool = False
     n_valid: int | None = None  # rows >= n_valid of X (and dY) are zero: token-axis zero padding
     description: str = ""
+    gains: str = "full"   # "full": G [N, C]; "separable": log gains g_t [N], g_c [C] (Eq. 2-3)
 
     @property
     def L(self) -> int:
@@ -101,7 +103,7 @@ class Workload:
         bwd = self.backward if backward is None else backward
         es = 2 if self.dtype == "bf16" else 4
         plane = self.B * self.L * es
-        g = self.L * 4
+        g = self.L * 4 if self.gains == "full" else (self.N + self.C) * 4
         fwd = 2 * plane + g
         if not bwd:
             return fwd
@@ -123,6 +125,10 @@ WORKLOADS = {
                                            description="two 135x240 maps, zero-padded to 65536 tokens, forward"),
     "train_16x8192x256_bf16": Workload("train_16x8192x256_bf16", 16, 8192, 256, "bf16", backward=True,
                                        description="training step: forward + backward"),
+    # the full-image shape with the paper's own gain form (Section III-B, Eq. 2-3): no G plane
+    "fullimage_separable_1x65536x128_bf16": Workload("fullimage_separable_1x65536x128_bf16", 1, 65536, 128, "bf16",
+                                                     n_valid=2 * 135 * 240, gains="separable",
+                                                     description="full-image shape, separable log gains, forward"),
 }
 WORKLOAD_ORDER = list(WORKLOADS)
 
@@ -166,8 +172,19 @@ def make_inputs(B: int, N: int, C: int, dtype: str, seed: int = 0, *, n_valid: i
     return out
 
 
+def make_log_gains(N: int, C: int, seed: int = 0, std: float = 0.05) -> tuple[np.ndarray, np.ndarray]:
+    """Separable log gains g_t [N], g_c [C] (float32 ~ N(0, std)): near the paper's zero
+    initialisation (unit gains), with a spread so that a wrong token or channel index is visible."""
+    g_t = normal(seed + 3, N, 0.0, std).astype(np.float32)
+    g_c = normal(seed + 4, C, 0.0, std).astype(np.float32)
+    return g_t, g_c
+
+
 def workload_inputs(w: Workload, seed: int = 0) -> dict[str, np.ndarray]:
-    return make_inputs(w.B, w.N, w.C, w.dtype, seed, n_valid=w.n_valid, with_dy=w.backward)
+    d = make_inputs(w.B, w.N, w.C, w.dtype, seed, n_valid=w.n_valid, with_dy=w.backward)
+    if w.gains == "separable":
+        d["g_t"], d["g_c"] = make_log_gains(w.N, w.C, seed)
+    return d
 
 
 def as_float64(a: np.ndarray, dtype: str) -> np.ndarray:

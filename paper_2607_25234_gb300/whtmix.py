@@ -17,8 +17,9 @@ import torch
 
 from . import build as _build
 
-__all__ = ["forward", "backward", "forward_ex", "backward_ex", "workspace_bytes", "sync", "plan",
-           "release_workspaces", "WhtmixError", "WHTMixFunction", "pad_tokens", "EXPORTS", "library"]
+__all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_separable", "backward_separable",
+           "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
+           "WHTMixSeparableFunction", "pad_tokens", "EXPORTS", "library"]
 
 # status codes and dtype codes of include/whtmix.h
 OK = 0
@@ -30,7 +31,8 @@ GAIN_DTYPE = {torch.float32: torch.float32, torch.bfloat16: torch.float32, torch
 # every entry point include/whtmix.h declares
 EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmix_forward_ex",
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
-           "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc")
+           "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc", "whtmix_forward_separable",
+           "whtmix_backward_separable")
 
 
 class WhtmixError(RuntimeError):
@@ -64,6 +66,8 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_status_string.restype = ctypes.c_char_p
             lib.whtmix_last_cuda_error.argtypes = []
             lib.whtmix_plan.argtypes = [i64, i64]
+            lib.whtmix_forward_separable.argtypes = [p, p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_backward_separable.argtypes = [p, p, p, p, p, p, p, i64, i64, i64, i, p]
             for name in EXPORTS:
                 if name != "whtmix_status_string":
                     getattr(lib, name).restype = ctypes.c_int
@@ -131,6 +135,52 @@ def backward(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torch.Tenso
     return dx, dg
 
 
+def _check_log_gains(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, *others: torch.Tensor):
+    if x.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError(f"separable gains need float32 or bfloat16 inputs, got {x.dtype}")
+    B, N, C = _shape(x)
+    if g_t.dtype != torch.float32 or g_c.dtype != torch.float32:
+        raise TypeError("log gains must be float32")
+    if tuple(g_t.shape) != (N,) or tuple(g_c.shape) != (C,):
+        raise ValueError(f"log gains must be g_t [{N}] and g_c [{C}], got {tuple(g_t.shape)} and {tuple(g_c.shape)}")
+    for t in (x, g_t, g_c) + others:
+        if not t.is_cuda:
+            raise ValueError("WHTMix runs on CUDA tensors only")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    return B, N, C
+
+
+def forward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, out: torch.Tensor | None = None,
+                      stream=None) -> torch.Tensor:
+    """The forward with the paper's log-domain gains (Section III-B, Eq. 2-3):
+    G[n, c] = exp(g_t[n]) exp(g_c[c])."""
+    B, N, C = _check_log_gains(x, g_t, g_c)
+    y = torch.empty_like(x) if out is None else out
+    if y.shape != x.shape or y.dtype != x.dtype:
+        raise ValueError("out must match x in shape and dtype")
+    _check(library().whtmix_forward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), y.data_ptr(), B, N, C,
+                                              DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_forward_separable")
+    return y
+
+
+def backward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, dy: torch.Tensor,
+                       dx: torch.Tensor | None = None, dg_t: torch.Tensor | None = None,
+                       dg_c: torch.Tensor | None = None, stream=None):
+    """(dX, dg_t, dg_c) of forward_separable."""
+    B, N, C = _check_log_gains(x, g_t, g_c, dy)
+    if dy.shape != x.shape or dy.dtype != x.dtype:
+        raise ValueError("dy must match x in shape and dtype")
+    dx = torch.empty_like(dy) if dx is None else dx
+    dg_t = torch.empty_like(g_t) if dg_t is None else dg_t
+    dg_c = torch.empty_like(g_c) if dg_c is None else dg_c
+    _check(library().whtmix_backward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), dy.data_ptr(),
+                                               dx.data_ptr(), dg_t.data_ptr(), dg_c.data_ptr(), B, N, C,
+                                               DTYPE_CODE[x.dtype], _stream_ptr(stream)),
+           "whtmix_backward_separable")
+    return dx, dg_t, dg_c
+
+
 def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool = False) -> int:
     out = ctypes.c_size_t(0)
     _check(library().whtmix_workspace_bytes(B, N, C, DTYPE_CODE[dtype], int(backward), ctypes.byref(out)),
@@ -195,3 +245,17 @@ class WHTMixFunction(torch.autograd.Function):
         x, g = ctx.saved_tensors
         dx, dg = backward(x, g, dy.contiguous())
         return dx, dg
+
+
+class WHTMixSeparableFunction(torch.autograd.Function):
+    """autograd wrapper for the log-domain gains: forward and backward both run in the CUDA library."""
+
+    @staticmethod
+    def forward(ctx, x, g_t, g_c):
+        ctx.save_for_backward(x, g_t, g_c)
+        return forward_separable(x.contiguous(), g_t.contiguous(), g_c.contiguous())
+
+    @staticmethod
+    def backward(ctx, dy):
+        x, g_t, g_c = ctx.saved_tensors
+        return backward_separable(x, g_t, g_c, dy.contiguous())

@@ -130,3 +130,34 @@ def test_no_device_reported_on_a_cpu_box(lib):
     if torch.cuda.is_available():
         pytest.skip("a GPU is present")
     assert fwd(lib) == 8
+
+
+def sfwd(lib, x=FAKE, gt=2 * FAKE, gc=2 * FAKE + 64, y=3 * FAKE, B=1, N=4, C=4, dtype=0):
+    return lib.whtmix_forward_separable(x, gt, gc, y, B, N, C, dtype, None)
+
+
+def sbwd(lib, x=FAKE, gt=2 * FAKE, gc=2 * FAKE + 64, dy=3 * FAKE, dx=4 * FAKE, dgt=5 * FAKE, dgc=5 * FAKE + 64,
+         B=1, N=4, C=4, dtype=0):
+    return lib.whtmix_backward_separable(x, gt, gc, dy, dx, dgt, dgc, B, N, C, dtype, None)
+
+
+def test_separable_rejects_invalid_arguments_before_any_device_work(lib):
+    assert sfwd(lib, dtype=2) == 3                    # int32: log-domain gains are real
+    assert sbwd(lib, dtype=2) == 3
+    assert sfwd(lib, gt=None) == 1
+    assert sfwd(lib, gc=None) == 1
+    assert sbwd(lib, dgt=None) == 1
+    assert sbwd(lib, dgc=None) == 1
+    assert sfwd(lib, N=6) == 2
+    assert sfwd(lib, x=FAKE + 8) == 4
+    assert sfwd(lib, gt=2 * FAKE + 2) == 4            # gains need 4-byte alignment only
+    assert sbwd(lib, dgc=5 * FAKE + 66) == 4
+    assert sfwd(lib, y=FAKE + 16) == 5                # partial overlap with x
+    assert sfwd(lib, y=2 * FAKE - 16) == 5            # output over g_t
+    assert sbwd(lib, dgt=FAKE + 16) == 5              # dg_t inside x
+    assert sbwd(lib, dgc=5 * FAKE + 8) == 5           # dg_c over dg_t
+    assert sbwd(lib, dx=FAKE) == 5                    # dx over x
+    # gains 4-byte aligned and exact in-place pass the host checks and stop at the device
+    assert sfwd(lib, gt=2 * FAKE + 4, y=FAKE) in (0, 6, 8)
+    assert sbwd(lib, dx=3 * FAKE) in (0, 6, 8)
+    assert sfwd(lib, B=0) == 0

@@ -171,6 +171,45 @@ def test_rank1_gain_equals_sequential_channel_then_token_mix(N, C):
     np.testing.assert_allclose(oracle.forward(x, np.outer(np.exp(g_t), np.exp(g_c))), z, rtol=1e-11, atol=1e-12)
 
 
+@pytest.mark.parametrize("N,C", [(4, 8), (32, 16), (16, 64)])
+def test_separable_forward_equals_sequential_eq2_then_eq3(N, C):
+    # forward_separable against the paper's sequential form written with dense orthonormal
+    # matrices: the channel mix with diag(exp(g_c)) on every token row (Eq. 2), then the token
+    # mix with diag(exp(g_t)) on every channel column (Eq. 3).
+    x = rng_normal((2, N, C), 15)
+    g_t, g_c = 0.2 * rng_normal((N,), 16), 0.2 * rng_normal((C,), 17)
+    hc = scipy.linalg.hadamard(C) / np.sqrt(C)
+    hn = scipy.linalg.hadamard(N) / np.sqrt(N)
+    want = np.stack([hn @ np.diag(np.exp(g_t)) @ hn @ (xb @ hc @ np.diag(np.exp(g_c)) @ hc) for xb in x])
+    np.testing.assert_allclose(oracle.forward_separable(x, g_t, g_c), want, rtol=1e-11, atol=1e-12)
+    # zero log gains are the paper's initialisation: the mixer starts as the identity
+    np.testing.assert_allclose(oracle.forward_separable(x, np.zeros(N), np.zeros(C)), x, rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("B,N,C", [(1, 8, 4), (3, 16, 8), (2, 4, 32)])
+def test_separable_backward_finite_differences(B, N, C):
+    x, dy = rng_normal((B, N, C), 45), rng_normal((B, N, C), 46)
+    g_t, g_c = 0.2 * rng_normal((N,), 47), 0.2 * rng_normal((C,), 48)
+    dx, dgt, dgc = oracle.backward_separable(x, g_t, g_c, dy)
+    np.testing.assert_allclose(dx, dense_forward(dy, np.outer(np.exp(g_t), np.exp(g_c))), rtol=1e-11, atol=1e-12)
+    loss = lambda gt, gc: np.vdot(oracle.forward_separable(x, gt, gc), dy)
+    eps = 1e-5
+    for n in sorted({0, N // 2, N - 1}):
+        e = np.zeros(N)
+        e[n] = eps
+        fd = (loss(g_t + e, g_c) - loss(g_t - e, g_c)) / (2 * eps)
+        assert abs(fd - dgt[n]) <= 1e-7 * max(1.0, abs(fd)), (n, fd, dgt[n])
+    for c in sorted({0, C // 2, C - 1}):
+        e = np.zeros(C)
+        e[c] = eps
+        fd = (loss(g_t, g_c + e) - loss(g_t, g_c - e)) / (2 * eps)
+        assert abs(fd - dgc[c]) <= 1e-7 * max(1.0, abs(fd)), (c, fd, dgc[c])
+    # a common shift of every log gain scales G by exp(s), so d loss / d s = loss = sum dg_t = sum dg_c
+    total = loss(g_t, g_c)
+    assert abs(dgt.sum() - total) <= 1e-10 * max(1.0, abs(total))
+    assert abs(dgc.sum() - total) <= 1e-10 * max(1.0, abs(total))
+
+
 def test_linear_in_x_and_in_g():
     N, C = 32, 16
     x1, x2 = rng_normal((N, C), 20), rng_normal((N, C), 21)
