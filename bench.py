@@ -275,7 +275,7 @@ def ours(args, w):
     def step(i):
         a = args_c[i % nsets]
         if sep:
-            rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, w.N, w.C, code, sp)
+            rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, w.N, w.N, w.C, code, sp)
         else:
             rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
         if rc != 0:

@@ -129,27 +129,43 @@ WHTMIX_API int whtmix_backward_ex(const void *x, const void *gains, const void *
 WHTMIX_API int whtmix_forward_noalloc(const void *x, const void *gains, void *y, int64_t B, int64_t N,
                                       int64_t C, int dtype, void *stream);
 
+/* Token-axis zero padding inside the library (Section III-B: a non-power-of-two token count is
+ * zero-padded to a power of two before H_N, and the padded outputs are discarded).  x, y, dy and
+ * dx hold only the first N_valid tokens of each plane, [B, N_valid, C] row-major; the mixer acts on
+ * the plane padded with zero rows to [N, C] (N a power of two, 0 <= N_valid <= N) and gains /
+ * dgains are [N, C].  Same results as padding by hand, calling whtmix_forward / whtmix_backward
+ * and cropping the output rows (the upstream gradient of the discarded rows is zero).  The fast
+ * kernels read only the stored rows and write only the kept rows when every stored plane starts
+ * 16-byte aligned (N_valid * C * sizeof(dtype) a multiple of 16); other shapes pad and crop through
+ * copies in the library workspace.  N_valid = N is exactly whtmix_forward / whtmix_backward;
+ * N_valid = 0 or B = 0 stores nothing (the backward sets dgains to zero).  Other rules as for
+ * whtmix_forward / whtmix_backward. */
+WHTMIX_API int whtmix_forward_padded(const void *x, const void *gains, void *y, int64_t B, int64_t N_valid, int64_t N,
+                                     int64_t C, int dtype, void *stream);
+WHTMIX_API int whtmix_backward_padded(const void *x, const void *gains, const void *dy, void *dx, void *dgains,
+                                      int64_t B, int64_t N_valid, int64_t N, int64_t C, int dtype, void *stream);
+
 /* The paper's own gain parameterisation (Section III-B, Eq. 2-3): per-frequency log gains for the
  * token axis, g_t [N], and the channel axis, g_c [C], fp32, applied in the WHT domain as
  * G[n, c] = exp(g_t[n]) * exp(g_c[c]).  Because the channel and token mixes act on different axes,
  * the sequential Eq. 2 -> Eq. 3 form equals the 2D map with this rank-one G, and these calls
- * compute exactly what whtmix_forward / whtmix_backward compute with
- * G = fp32(expf(g_t[n]) * expf(g_c[c])).  dtype is WHTMIX_F32 or WHTMIX_BF16 (WHTMIX_I32 returns
- * WHTMIX_ERR_BAD_DTYPE).  x, y, dy, dx: 16-byte aligned; g_t, g_c, dg_t, dg_c: 4-byte aligned,
- * device memory owned by the caller.
+ * compute exactly what whtmix_forward_padded / whtmix_backward_padded compute with
+ * G = fp32(expf(g_t[n]) * expf(g_c[c])), token padding included (N_valid as there; N_valid = N for
+ * none).  dtype is WHTMIX_F32 or WHTMIX_BF16 (WHTMIX_I32 returns WHTMIX_ERR_BAD_DTYPE).  x, y, dy,
+ * dx: 16-byte aligned; g_t, g_c, dg_t, dg_c: 4-byte aligned; device memory owned by the caller.
  * Forward: for the planes the fast kernel covers (2^14 <= N*C <= 2^23) with 2 <= C <= 2^13 (2^14
  * for N*C = 2^23), the gains are computed inside the kernel from two small tables of exp values
  * and G never exists in memory; other shapes build G in the library workspace first.
- * Backward: dx as whtmix_backward with that G; dg_t[n] = sum_c dG[n, c] G[n, c] and
+ * Backward: dx as whtmix_backward_padded with that G; dg_t[n] = sum_c dG[n, c] G[n, c] and
  * dg_c[c] = sum_n dG[n, c] G[n, c] with dG = sum_b (W X_b) o (W dY_b) (the chain rule through
- * the exponentials), each a fixed-order sum (bit-reproducible).  dg_t and dg_c are overwritten.
- * B = 0: the forward is a no-op; the backward sets dg_t and dg_c to zero.
- * Aliasing as for whtmix_forward / whtmix_backward (y == x and dx == dy allowed). */
+ * the exponentials), each a fixed-order sum accumulated in float64 (bit-reproducible).  dg_t and
+ * dg_c are overwritten.  B = 0 or N_valid = 0: the forward is a no-op; the backward sets dg_t and
+ * dg_c to zero.  Aliasing as for whtmix_forward / whtmix_backward (y == x and dx == dy allowed). */
 WHTMIX_API int whtmix_forward_separable(const void *x, const float *g_t, const float *g_c, void *y, int64_t B,
-                                        int64_t N, int64_t C, int dtype, void *stream);
+                                        int64_t N_valid, int64_t N, int64_t C, int dtype, void *stream);
 WHTMIX_API int whtmix_backward_separable(const void *x, const float *g_t, const float *g_c, const void *dy, void *dx,
-                                         float *dg_t, float *dg_c, int64_t B, int64_t N, int64_t C, int dtype,
-                                         void *stream);
+                                         float *dg_t, float *dg_c, int64_t B, int64_t N_valid, int64_t N, int64_t C,
+                                         int dtype, void *stream);
 
 /* Synchronises `stream` and reports device-side failures of the calls enqueued on it since the
  * previous whtmix_sync: WHTMIX_ERR_TIMEOUT if a bounded device-wide wait gave up (the library

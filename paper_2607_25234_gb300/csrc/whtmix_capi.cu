@@ -227,77 +227,6 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
   return launch(k_backward_m<D>, true, sms, 2ll * (static_cast<long long>(P.gp) << (m - TILE_BITS)), 3 * tile_bytes, P, stream);
 }
 
-int run(bool backward, const void* x, const void* g, const void* dy, void* y_or_dx, void* dg,
-        int64_t B, int64_t N, int64_t C, int dtype, void* user_ws, size_t user_ws_bytes, bool use_user_ws,
-        void* stream_v) {
-  int m = 0;
-  int rc = check_shape(B, N, C, dtype, &m);
-  if (rc != WHTMIX_OK) return rc;
-  if (B == 0) {
-    // Empty batch: the forward has nothing to do (any pointers, even null, are accepted); the
-    // backward's dG is a sum over no planes, so it is set to zero.
-    if (!backward) return WHTMIX_OK;
-    if (!dg) return WHTMIX_ERR_INVALID_ARG;
-    if (!aligned16(dg)) return WHTMIX_ERR_MISALIGNED;
-    int dev = 0, sms = 0;
-    rc = device_check(&dev, &sms);
-    if (rc != WHTMIX_OK) return rc;
-    cudaError_t e = cudaMemsetAsync(dg, 0, (size_t{1} << m) * 4, static_cast<cudaStream_t>(stream_v));
-    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
-  }
-  if (!x || !g || !y_or_dx || (backward && (!dy || !dg))) return WHTMIX_ERR_INVALID_ARG;
-  if (!aligned16(x) || !aligned16(g) || !aligned16(y_or_dx) || (backward && (!aligned16(dy) || !aligned16(dg))))
-    return WHTMIX_ERR_MISALIGNED;
-  const size_t L = size_t{1} << m;
-  const size_t plane_bytes = static_cast<size_t>(B) * L * elem_size(dtype);
-  const size_t g_bytes = L * 4;
-  if (!backward) {
-    if (y_or_dx != x && overlap(y_or_dx, plane_bytes, x, plane_bytes)) return WHTMIX_ERR_ALIAS;
-    if (overlap(y_or_dx, plane_bytes, g, g_bytes)) return WHTMIX_ERR_ALIAS;
-  } else {
-    void* dx = y_or_dx;
-    if (dx != dy && overlap(dx, plane_bytes, dy, plane_bytes)) return WHTMIX_ERR_ALIAS;
-    if (overlap(dx, plane_bytes, x, plane_bytes) || overlap(dx, plane_bytes, g, g_bytes)) return WHTMIX_ERR_ALIAS;
-    if (overlap(dg, g_bytes, x, plane_bytes) || overlap(dg, g_bytes, dy, plane_bytes) ||
-        overlap(dg, g_bytes, dx, plane_bytes) || overlap(dg, g_bytes, g, g_bytes))
-      return WHTMIX_ERR_ALIAS;
-  }
-  const size_t need = workspace_bytes(B, m, backward);
-  if (use_user_ws) {
-    if (!user_ws || (reinterpret_cast<uintptr_t>(user_ws) & 255u) || user_ws_bytes < need) return WHTMIX_ERR_WORKSPACE;
-  }
-  int dev = 0, sms = 0;
-  rc = device_check(&dev, &sms);
-  if (rc != WHTMIX_OK) return rc;
-  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
-  void* ws = user_ws;
-  if (!use_user_ws) {
-    rc = cached_workspace(dev, stream, need, &ws);
-    if (rc != WHTMIX_OK) return rc;
-  }
-  Params P{};
-  P.x = x;
-  P.g = g;
-  P.dy = dy;
-  if (backward) {
-    P.dx = y_or_dx;
-    P.dg = dg;
-  } else {
-    P.y = y_or_dx;
-  }
-  P.bar = static_cast<GridBarrier*>(ws);
-  P.ws = static_cast<char*>(ws) + HEADER_BYTES;
-  P.B = B;
-  P.m = m;
-  P.gp = planes_per_group(B, m, backward);
-  P.scale = 1.0f / static_cast<float>(L);
-  switch (dtype) {
-    case WHTMIX_F32: return dispatch<DT_F32>(backward, P, sms, stream);
-    case WHTMIX_BF16: return dispatch<DT_BF16>(backward, P, sms, stream);
-    default: return dispatch<DT_I32>(backward, P, sms, stream);
-  }
-}
-
 // ---- separable log gains (Section III-B, Eq. 2-3): G[n, c] = exp(g_t[n]) exp(g_c[c]) ----
 
 constexpr int SEP_THREADS = 256;
@@ -374,105 +303,285 @@ bool use_fast_separable(int dtype, int m, int cbits) {
   return use_fast_forward(dtype, m) && cbits >= 1 && cbits <= fast::forward_row_bits(m);
 }
 
-size_t separable_workspace_bytes(int64_t B, int m, int cbits, int dtype, bool backward) {
-  const size_t base = align256(workspace_bytes(B, m, backward));
-  const size_t L = size_t{1} << m;
-  if (!backward) {
-    if (use_fast_separable(dtype, m, cbits)) return base + align256(((L >> cbits) + (size_t{1} << cbits)) * 4);
-    return base + align256(L * 4);
+// Zero padding / crop on the token axis for the shapes the fast kernels do not pad themselves:
+// planes of lv stored elements <-> planes of 2^m elements (element size es bytes).
+__global__ void k_pad_planes(void* dst, const void* src, long long B, long long lv, int m, int es) {
+  const long long L = 1ll << m;
+  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < B * L;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long b = i >> m, e = i & (L - 1);
+    if (es == 2)
+      static_cast<unsigned short*>(dst)[i] = e < lv ? static_cast<const unsigned short*>(src)[b * lv + e] : 0;
+    else
+      static_cast<unsigned int*>(dst)[i] = e < lv ? static_cast<const unsigned int*>(src)[b * lv + e] : 0u;
   }
-  return base + 2 * align256(L * 4) + align256(static_cast<size_t>(sep_chunks(m, cbits) << cbits) * 8);
+}
+__global__ void k_crop_planes(void* dst, const void* src, long long B, long long lv, int m, int es) {
+  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < B * lv;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long b = i / lv, e = i - b * lv;
+    if (es == 2)
+      static_cast<unsigned short*>(dst)[i] = static_cast<const unsigned short*>(src)[(b << m) + e];
+    else
+      static_cast<unsigned int*>(dst)[i] = static_cast<const unsigned int*>(src)[(b << m) + e];
+  }
 }
 
-int run_separable(bool backward, const void* x, const float* gt, const float* gc, const void* dy, void* y_or_dx,
-                  float* dgt, float* dgc, int64_t B, int64_t N, int64_t C, int dtype, void* stream_v) {
+// One call of the C ABI, after its arguments are named: full gains (g, dg) or separable log gains
+// (gt, gc, dgt, dgc); x, y / dx and dy hold n_valid of the N rows of each plane.
+struct Call {
+  bool backward = false;
+  bool separable = false;
+  const void* x = nullptr;
+  const void* g = nullptr;
+  const float* gt = nullptr;
+  const float* gc = nullptr;
+  const void* dy = nullptr;
+  void* out = nullptr;  // y (forward) or dx (backward)
+  void* dg = nullptr;
+  float* dgt = nullptr;
+  float* dgc = nullptr;
+  int64_t B = 0, n_valid = 0, N = 0, C = 0;
+  int dtype = 0;
+};
+
+// Workspace layout of a call: the kernel workspace (barrier header + plane group) first, then
+// the separable tables or G / dG / partial sums, then the zero-padded copies.
+struct Layout {
+  size_t base = 0, g = 0, dg = 0, part = 0, pad = 0, total = 0;
+  bool fast_sep = false, pad_copy = false;
+  int pad_planes = 0;
+};
+
+Layout plan_call(const Call& c, int m) {
+  Layout l;
+  const size_t L = size_t{1} << m;
+  const int cbits = ilog2_pow2(c.C);
+  const size_t es = elem_size(c.dtype);
+  const size_t lv = static_cast<size_t>(c.n_valid) * static_cast<size_t>(c.C);
+  // the fast kernels pad and crop in their row passes when every stored plane starts 16-byte aligned
+  const bool fast = c.backward ? use_fast_backward(c.dtype, m) : use_fast_forward(c.dtype, m);
+  l.pad_copy = lv < L && !(fast && (lv * es) % 16 == 0);
+  l.fast_sep = c.separable && !c.backward && !l.pad_copy && use_fast_separable(c.dtype, m, cbits);
+  l.base = workspace_bytes(c.B, m, c.backward);  // exactly whtmix_workspace_bytes for a plain call
+  size_t off = l.base;
+  if (c.separable || l.pad_copy) off = align256(off);
+  if (l.fast_sep) {
+    off += align256((L >> cbits) * 4 + (size_t{1} << cbits) * 4);  // exp tables, right after the plane group
+  } else if (c.separable) {
+    l.g = off;
+    off += align256(L * 4);
+    if (c.backward) {
+      l.dg = off;
+      off += align256(L * 4);
+      l.part = off;
+      off += align256(static_cast<size_t>(sep_chunks(m, cbits) << cbits) * 8);
+    }
+  }
+  if (l.pad_copy) {
+    l.pad = off;
+    l.pad_planes = c.backward ? 3 : 2;  // x, y  |  x, dy, dx
+    off += l.pad_planes * align256(static_cast<size_t>(c.B) * L * es);
+  }
+  l.total = off;
+  return l;
+}
+
+int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, void* stream_v) {
   int m = 0;
-  int rc = check_shape(B, N, C, dtype, &m);
+  int rc = check_shape(c.B, c.N, c.C, c.dtype, &m);
   if (rc != WHTMIX_OK) return rc;
-  if (dtype == WHTMIX_I32) return WHTMIX_ERR_BAD_DTYPE;  // log-domain gains are real
-  const int cbits = ilog2_pow2(C);
+  if (c.n_valid < 0 || c.n_valid > c.N) return WHTMIX_ERR_INVALID_ARG;
+  if (c.separable && c.dtype == WHTMIX_I32) return WHTMIX_ERR_BAD_DTYPE;  // log-domain gains are real
   cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  const size_t L = size_t{1} << m;
+  const size_t es = elem_size(c.dtype);
+  const size_t lv = static_cast<size_t>(c.n_valid) * static_cast<size_t>(c.C);
+  const size_t plane_bytes = static_cast<size_t>(c.B) * lv * es;
+  const size_t g_bytes = L * 4, t_bytes = static_cast<size_t>(c.N) * 4, ch_bytes = static_cast<size_t>(c.C) * 4;
   auto aligned4 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; };
-  const size_t N_bytes = static_cast<size_t>(N) * 4, C_bytes = static_cast<size_t>(C) * 4;
-  if (B == 0) {
-    // Empty batch: the forward has nothing to do; the backward's gradients are sums over no planes.
-    if (!backward) return WHTMIX_OK;
-    if (!dgt || !dgc) return WHTMIX_ERR_INVALID_ARG;
-    if (!aligned4(dgt) || !aligned4(dgc)) return WHTMIX_ERR_MISALIGNED;
-    if (overlap(dgt, N_bytes, dgc, C_bytes)) return WHTMIX_ERR_ALIAS;
+  if (c.B == 0 || lv == 0) {
+    // No stored elements: the forward has nothing to do (any pointers, even null, are accepted);
+    // the backward's gain gradients are sums over nothing, so they are set to zero.
+    if (!c.backward) return WHTMIX_OK;
+    if (c.separable) {
+      if (!c.dgt || !c.dgc) return WHTMIX_ERR_INVALID_ARG;
+      if (!aligned4(c.dgt) || !aligned4(c.dgc)) return WHTMIX_ERR_MISALIGNED;
+      if (overlap(c.dgt, t_bytes, c.dgc, ch_bytes)) return WHTMIX_ERR_ALIAS;
+    } else {
+      if (!c.dg) return WHTMIX_ERR_INVALID_ARG;
+      if (!aligned16(c.dg)) return WHTMIX_ERR_MISALIGNED;
+    }
     int dev = 0, sms = 0;
     rc = device_check(&dev, &sms);
     if (rc != WHTMIX_OK) return rc;
-    cudaError_t e = cudaMemsetAsync(dgt, 0, N_bytes, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(dgc, 0, C_bytes, stream);
+    cudaError_t e = c.separable ? cudaMemsetAsync(c.dgt, 0, t_bytes, stream) : cudaMemsetAsync(c.dg, 0, g_bytes, stream);
+    if (e == cudaSuccess && c.separable) e = cudaMemsetAsync(c.dgc, 0, ch_bytes, stream);
     return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
   }
-  if (!x || !gt || !gc || !y_or_dx || (backward && (!dy || !dgt || !dgc))) return WHTMIX_ERR_INVALID_ARG;
-  if (!aligned16(x) || !aligned16(y_or_dx) || (backward && !aligned16(dy))) return WHTMIX_ERR_MISALIGNED;
-  if (!aligned4(gt) || !aligned4(gc) || (backward && (!aligned4(dgt) || !aligned4(dgc)))) return WHTMIX_ERR_MISALIGNED;
-  const size_t L = size_t{1} << m;
-  const size_t plane_bytes = static_cast<size_t>(B) * L * elem_size(dtype);
-  void* out = y_or_dx;
-  const void* in = backward ? dy : x;
-  if (out != in && overlap(out, plane_bytes, in, plane_bytes)) return WHTMIX_ERR_ALIAS;
-  if (overlap(out, plane_bytes, gt, N_bytes) || overlap(out, plane_bytes, gc, C_bytes)) return WHTMIX_ERR_ALIAS;
-  if (backward) {
-    if (overlap(out, plane_bytes, x, plane_bytes)) return WHTMIX_ERR_ALIAS;
-    const void* ins[5] = {x, dy, gt, gc, out};
-    const size_t ins_bytes[5] = {plane_bytes, plane_bytes, N_bytes, C_bytes, plane_bytes};
-    for (int i = 0; i < 5; ++i)
-      if (overlap(dgt, N_bytes, ins[i], ins_bytes[i]) || overlap(dgc, C_bytes, ins[i], ins_bytes[i]))
-        return WHTMIX_ERR_ALIAS;
-    if (overlap(dgt, N_bytes, dgc, C_bytes)) return WHTMIX_ERR_ALIAS;
+  // pointers, alignment, aliasing
+  if (!c.x || !c.out || (c.backward && !c.dy)) return WHTMIX_ERR_INVALID_ARG;
+  if (c.separable ? (!c.gt || !c.gc || (c.backward && (!c.dgt || !c.dgc))) : (!c.g || (c.backward && !c.dg)))
+    return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(c.x) || !aligned16(c.out) || (c.backward && !aligned16(c.dy))) return WHTMIX_ERR_MISALIGNED;
+  if (c.separable) {
+    if (!aligned4(c.gt) || !aligned4(c.gc) || (c.backward && (!aligned4(c.dgt) || !aligned4(c.dgc))))
+      return WHTMIX_ERR_MISALIGNED;
+  } else if (!aligned16(c.g) || (c.backward && !aligned16(c.dg))) {
+    return WHTMIX_ERR_MISALIGNED;
+  }
+  // read-only inputs the output must not touch; the output may equal its own input exactly
+  const void* in = c.backward ? c.dy : c.x;
+  if (c.out != in && overlap(c.out, plane_bytes, in, plane_bytes)) return WHTMIX_ERR_ALIAS;
+  const void* ro[4];
+  size_t ro_bytes[4];
+  int nro = 0;
+  if (c.separable) {
+    ro[nro] = c.gt, ro_bytes[nro++] = t_bytes;
+    ro[nro] = c.gc, ro_bytes[nro++] = ch_bytes;
+  } else {
+    ro[nro] = c.g, ro_bytes[nro++] = g_bytes;
+  }
+  if (c.backward) ro[nro] = c.x, ro_bytes[nro++] = plane_bytes;
+  for (int i = 0; i < nro; ++i)
+    if (overlap(c.out, plane_bytes, ro[i], ro_bytes[i])) return WHTMIX_ERR_ALIAS;
+  if (c.backward) {
+    // gain gradients: disjoint from every other buffer of the call
+    const void* all[6] = {c.x, c.dy, c.out, c.separable ? static_cast<const void*>(c.gt) : c.g, c.gc, c.dgc};
+    const size_t all_bytes[6] = {plane_bytes, plane_bytes, plane_bytes, c.separable ? t_bytes : g_bytes,
+                                 c.separable ? ch_bytes : 0, c.separable ? ch_bytes : 0};
+    const void* gout = c.separable ? static_cast<const void*>(c.dgt) : c.dg;
+    const size_t gout_bytes = c.separable ? t_bytes : g_bytes;
+    for (int i = 0; i < 6; ++i)
+      if (overlap(gout, gout_bytes, all[i], all_bytes[i])) return WHTMIX_ERR_ALIAS;
+    if (c.separable)
+      for (int i = 0; i < 5; ++i)
+        if (overlap(c.dgc, ch_bytes, all[i], all_bytes[i])) return WHTMIX_ERR_ALIAS;
+  }
+  const Layout lay = plan_call(c, m);
+  if (use_user_ws) {
+    if (!user_ws || (reinterpret_cast<uintptr_t>(user_ws) & 255u) || user_ws_bytes < lay.total) return WHTMIX_ERR_WORKSPACE;
   }
   int dev = 0, sms = 0;
   rc = device_check(&dev, &sms);
   if (rc != WHTMIX_OK) return rc;
-  void* ws = nullptr;
-  rc = cached_workspace(dev, stream, separable_workspace_bytes(B, m, cbits, dtype, backward), &ws);
-  if (rc != WHTMIX_OK) return rc;
-  char* extra = static_cast<char*>(ws) + align256(workspace_bytes(B, m, backward));
+  void* ws = user_ws;
+  if (!use_user_ws) {
+    rc = cached_workspace(dev, stream, lay.total, &ws);
+    if (rc != WHTMIX_OK) return rc;
+  }
+  char* wsb = static_cast<char*>(ws);
+  const int cbits = ilog2_pow2(c.C);
   Params P{};
-  P.x = x;
-  P.dy = dy;
+  P.x = c.x;
+  P.g = c.g;
+  P.dy = c.dy;
+  if (c.backward) {
+    P.dx = c.out;
+    P.dg = c.dg;
+  } else {
+    P.y = c.out;
+  }
   P.bar = static_cast<GridBarrier*>(ws);
-  P.ws = static_cast<char*>(ws) + HEADER_BYTES;
-  P.B = B;
+  P.ws = wsb + HEADER_BYTES;
+  P.B = c.B;
   P.m = m;
-  P.gp = planes_per_group(B, m, backward);
+  P.gp = planes_per_group(c.B, m, c.backward);
   P.scale = 1.0f / static_cast<float>(L);
-  P.gt = gt;
-  P.gc = gc;
+  P.gt = c.gt;
+  P.gc = c.gc;
   P.cbits = cbits;
-  if (!backward && use_fast_separable(dtype, m, cbits)) {
-    // the gain tables go right after the plane group, where the kernel expects them
-    P.y = y_or_dx;
-    const cudaError_t e = dtype == WHTMIX_BF16 ? fast::forward_sep_bf16(P, sms, stream) : fast::forward_sep_f32(P, sms, stream);
+  P.lv = static_cast<long long>(lv);
+  cudaError_t e = cudaSuccess;
+  if (lay.fast_sep) {
+    e = c.dtype == WHTMIX_BF16 ? fast::forward_sep_bf16(P, sms, stream) : fast::forward_sep_f32(P, sms, stream);
     return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
   }
-  // Otherwise G is built in the workspace and the full-gain kernels run on it.
-  float* G = reinterpret_cast<float*>(extra);
-  k_sep_gains<<<grid_for(static_cast<long long>(L), sms), SEP_THREADS, 0, stream>>>(G, gt, gc, m, cbits);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e);
-  P.g = G;
-  if (!backward) {
-    P.y = y_or_dx;
-    return dtype == WHTMIX_BF16 ? dispatch<DT_BF16>(false, P, sms, stream) : dispatch<DT_F32>(false, P, sms, stream);
+  if (c.separable) {
+    // the separable gains as a G plane in the workspace, for the full-gain kernels
+    float* G = reinterpret_cast<float*>(wsb + lay.g);
+    k_sep_gains<<<grid_for(static_cast<long long>(L), sms), SEP_THREADS, 0, stream>>>(G, c.gt, c.gc, m, cbits);
+    P.g = G;
+    if (c.backward) P.dg = wsb + lay.dg;
   }
-  float* dG = reinterpret_cast<float*>(extra + align256(L * 4));
-  double* part = reinterpret_cast<double*>(extra + 2 * align256(L * 4));
-  P.dx = y_or_dx;
-  P.dg = dG;
-  rc = dtype == WHTMIX_BF16 ? dispatch<DT_BF16>(true, P, sms, stream) : dispatch<DT_F32>(true, P, sms, stream);
+  void* out_pad = nullptr;
+  if (lay.pad_copy) {
+    const size_t pb = align256(static_cast<size_t>(c.B) * L * es);
+    void* xpad = wsb + lay.pad;
+    out_pad = wsb + lay.pad + pb;
+    const unsigned grid = grid_for(c.B * static_cast<long long>(L), sms);
+    k_pad_planes<<<grid, SEP_THREADS, 0, stream>>>(xpad, c.x, c.B, static_cast<long long>(lv), m, static_cast<int>(es));
+    P.x = xpad;
+    if (c.backward) {
+      void* dypad = wsb + lay.pad + 2 * pb;
+      k_pad_planes<<<grid, SEP_THREADS, 0, stream>>>(dypad, c.dy, c.B, static_cast<long long>(lv), m, static_cast<int>(es));
+      P.dy = dypad;
+      P.dx = out_pad;
+    } else {
+      P.y = out_pad;
+    }
+    P.lv = static_cast<long long>(L);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  switch (c.dtype) {
+    case WHTMIX_F32: rc = dispatch<DT_F32>(c.backward, P, sms, stream); break;
+    case WHTMIX_BF16: rc = dispatch<DT_BF16>(c.backward, P, sms, stream); break;
+    default: rc = dispatch<DT_I32>(c.backward, P, sms, stream); break;
+  }
   if (rc != WHTMIX_OK) return rc;
-  const long long nchunks = sep_chunks(m, cbits), Nn = 1ll << (m - cbits);
-  k_sep_reduce_t<<<grid_for(Nn * 32, sms), SEP_THREADS, 0, stream>>>(dgt, dG, G, m, cbits);
-  k_sep_reduce_c_part<<<grid_for(nchunks << cbits, sms), SEP_THREADS, 0, stream>>>(part, dG, G, m, cbits,
-                                                                                    (Nn + nchunks - 1) / nchunks, nchunks);
-  k_sep_reduce_c_final<<<grid_for(1ll << cbits, sms), SEP_THREADS, 0, stream>>>(dgc, part, cbits, nchunks);
+  if (lay.pad_copy)
+    k_crop_planes<<<grid_for(c.B * static_cast<long long>(lv), sms), SEP_THREADS, 0, stream>>>(
+        c.out, out_pad, c.B, static_cast<long long>(lv), m, static_cast<int>(es));
+  if (c.separable && c.backward) {
+    const float* G = static_cast<const float*>(P.g);
+    const float* dG = reinterpret_cast<const float*>(wsb + lay.dg);
+    double* part = reinterpret_cast<double*>(wsb + lay.part);
+    const long long nchunks = sep_chunks(m, cbits), Nn = 1ll << (m - cbits);
+    k_sep_reduce_t<<<grid_for(Nn * 32, sms), SEP_THREADS, 0, stream>>>(c.dgt, dG, G, m, cbits);
+    k_sep_reduce_c_part<<<grid_for(nchunks << cbits, sms), SEP_THREADS, 0, stream>>>(part, dG, G, m, cbits,
+                                                                                      (Nn + nchunks - 1) / nchunks, nchunks);
+    k_sep_reduce_c_final<<<grid_for(1ll << cbits, sms), SEP_THREADS, 0, stream>>>(c.dgc, part, cbits, nchunks);
+  }
   e = cudaGetLastError();
   return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+}
+
+Call full_call(bool backward, const void* x, const void* g, const void* dy, void* out, void* dg, int64_t B,
+               int64_t n_valid, int64_t N, int64_t C, int dtype) {
+  Call c;
+  c.backward = backward;
+  c.x = x;
+  c.g = g;
+  c.dy = dy;
+  c.out = out;
+  c.dg = dg;
+  c.B = B;
+  c.n_valid = n_valid;
+  c.N = N;
+  c.C = C;
+  c.dtype = dtype;
+  return c;
+}
+
+Call separable_call(bool backward, const void* x, const float* gt, const float* gc, const void* dy, void* out,
+                    float* dgt, float* dgc, int64_t B, int64_t n_valid, int64_t N, int64_t C, int dtype) {
+  Call c;
+  c.backward = backward;
+  c.separable = true;
+  c.x = x;
+  c.gt = gt;
+  c.gc = gc;
+  c.dy = dy;
+  c.out = out;
+  c.dgt = dgt;
+  c.dgc = dgc;
+  c.B = B;
+  c.n_valid = n_valid;
+  c.N = N;
+  c.C = C;
+  c.dtype = dtype;
+  return c;
 }
 
 }  // namespace
@@ -480,32 +589,46 @@ int run_separable(bool backward, const void* x, const float* gt, const float* gc
 extern "C" {
 
 int whtmix_forward(const void* x, const void* gains, void* y, int64_t B, int64_t N, int64_t C, int dtype, void* stream) {
-  return run(false, x, gains, nullptr, y, nullptr, B, N, C, dtype, nullptr, 0, false, stream);
+  return run(full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype), nullptr, 0, false, stream);
 }
 
 int whtmix_backward(const void* x, const void* gains, const void* dy, void* dx, void* dgains, int64_t B, int64_t N,
                     int64_t C, int dtype, void* stream) {
-  return run(true, x, gains, dy, dx, dgains, B, N, C, dtype, nullptr, 0, false, stream);
+  return run(full_call(true, x, gains, dy, dx, dgains, B, N, N, C, dtype), nullptr, 0, false, stream);
 }
 
 int whtmix_forward_ex(const void* x, const void* gains, void* y, int64_t B, int64_t N, int64_t C, int dtype,
                       void* workspace, size_t workspace_bytes_, void* stream) {
-  return run(false, x, gains, nullptr, y, nullptr, B, N, C, dtype, workspace, workspace_bytes_, true, stream);
+  return run(full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype), workspace, workspace_bytes_, true,
+             stream);
 }
 
 int whtmix_backward_ex(const void* x, const void* gains, const void* dy, void* dx, void* dgains, int64_t B, int64_t N,
                        int64_t C, int dtype, void* workspace, size_t workspace_bytes_, void* stream) {
-  return run(true, x, gains, dy, dx, dgains, B, N, C, dtype, workspace, workspace_bytes_, true, stream);
+  return run(full_call(true, x, gains, dy, dx, dgains, B, N, N, C, dtype), workspace, workspace_bytes_, true, stream);
 }
 
-int whtmix_forward_separable(const void* x, const float* g_t, const float* g_c, void* y, int64_t B, int64_t N,
-                             int64_t C, int dtype, void* stream) {
-  return run_separable(false, x, g_t, g_c, nullptr, y, nullptr, nullptr, B, N, C, dtype, stream);
+int whtmix_forward_padded(const void* x, const void* gains, void* y, int64_t B, int64_t N_valid, int64_t N, int64_t C,
+                          int dtype, void* stream) {
+  return run(full_call(false, x, gains, nullptr, y, nullptr, B, N_valid, N, C, dtype), nullptr, 0, false, stream);
+}
+
+int whtmix_backward_padded(const void* x, const void* gains, const void* dy, void* dx, void* dgains, int64_t B,
+                           int64_t N_valid, int64_t N, int64_t C, int dtype, void* stream) {
+  return run(full_call(true, x, gains, dy, dx, dgains, B, N_valid, N, C, dtype), nullptr, 0, false, stream);
+}
+
+int whtmix_forward_separable(const void* x, const float* g_t, const float* g_c, void* y, int64_t B, int64_t N_valid,
+                             int64_t N, int64_t C, int dtype, void* stream) {
+  return run(separable_call(false, x, g_t, g_c, nullptr, y, nullptr, nullptr, B, N_valid, N, C, dtype), nullptr, 0,
+             false, stream);
 }
 
 int whtmix_backward_separable(const void* x, const float* g_t, const float* g_c, const void* dy, void* dx,
-                              float* dg_t, float* dg_c, int64_t B, int64_t N, int64_t C, int dtype, void* stream) {
-  return run_separable(true, x, g_t, g_c, dy, dx, dg_t, dg_c, B, N, C, dtype, stream);
+                              float* dg_t, float* dg_c, int64_t B, int64_t N_valid, int64_t N, int64_t C, int dtype,
+                              void* stream) {
+  return run(separable_call(true, x, g_t, g_c, dy, dx, dg_t, dg_c, B, N_valid, N, C, dtype), nullptr, 0, false,
+             stream);
 }
 
 int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype, int backward, size_t* out_bytes) {

@@ -177,6 +177,8 @@ __device__ __forceinline__ void bfly_lane4(float2 (&b)[64]) {
 
 // Storage <-> fp32 for the two floating dtypes.
 template <int D> struct IOv;
+// (ld8_lim / st8_lim: only the first `n` of the 8 elements exist in memory, n a multiple of the
+// 16-byte chunk's element count; the others read as zero and are not written.)
 template <> struct IOv<DT_BF16> {
   // 8 consecutive elements at element index e (16-byte aligned): 4 pairs (r0 = 0, 1)
   __device__ static __forceinline__ void ld8(const void* p, long long e, float2 (&o)[4]) {
@@ -194,6 +196,9 @@ template <> struct IOv<DT_BF16> {
     }
     __stcs(reinterpret_cast<uint4*>(static_cast<unsigned short*>(p) + e), make_uint4(w[0], w[1], w[2], w[3]));
   }
+  __device__ static __forceinline__ void st8_lim(void* p, long long e, const float2 (&v)[4], long long n) {
+    if (n > 0) st8(p, e, v);
+  }
 };
 template <> struct IOv<DT_F32> {
   __device__ static __forceinline__ void ld8(const void* p, long long e, float2 (&o)[4]) {
@@ -209,6 +214,20 @@ template <> struct IOv<DT_F32> {
     __stcs(q, make_float4(v[0].x, v[0].y, v[1].x, v[1].y));
     __stcs(q + 1, make_float4(v[2].x, v[2].y, v[3].x, v[3].y));
   }
+  __device__ static __forceinline__ void ld8_lim(const void* p, long long e, float2 (&o)[4], long long n) {
+    const float4* q = reinterpret_cast<const float4*>(static_cast<const float*>(p) + e);
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 a = n > 0 ? __ldcs(q) : z, b = n > 4 ? __ldcs(q + 1) : z;
+    o[0] = make_float2(a.x, a.y);
+    o[1] = make_float2(a.z, a.w);
+    o[2] = make_float2(b.x, b.y);
+    o[3] = make_float2(b.z, b.w);
+  }
+  __device__ static __forceinline__ void st8_lim(void* p, long long e, const float2 (&v)[4], long long n) {
+    float4* q = reinterpret_cast<float4*>(static_cast<float*>(p) + e);
+    if (n > 0) __stcs(q, make_float4(v[0].x, v[0].y, v[1].x, v[1].y));
+    if (n > 4) __stcs(q + 1, make_float4(v[2].x, v[2].y, v[3].x, v[3].y));
+  }
 };
 
 // ---------------------------------------------------------------------------------------------
@@ -216,6 +235,11 @@ template <> struct IOv<DT_F32> {
 __device__ __forceinline__ void cp_async16(float* smem_dst, const void* gsrc) {
   const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gsrc) : "memory");
+}
+// 16-byte copy of which only the first src_bytes (0 or 16) are read; the rest is zero-filled.
+__device__ __forceinline__ void cp_async16_zfill(float* smem_dst, const void* gsrc, int src_bytes) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(gsrc), "r"(src_bytes) : "memory");
 }
 __device__ __forceinline__ void cp_async8(float* smem_dst, const void* gsrc) {
   const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
@@ -243,19 +267,26 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 // itself, so the staging area needs no barrier; chunk k of thread wt sits at (k * WORKER + wt),
 // which makes each warp's read-back one contiguous span.
 // Phase 1 stages a whole bf16 row (16 vectors of 8 elements) or the first half of an fp32 row.
+// Elements of the row at offsets >= lim are padding: not read, staged as zeros.
 template <int D, int R>
-__device__ __forceinline__ void stage_row_in(const void* src, long long e0, float* stg, int wt) {
+__device__ __forceinline__ void stage_row_in(const void* src, long long e0, float* stg, int wt, int lim) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   if constexpr (D == DT_BF16) {
 #pragma unroll
-    for (int v = 0; v < 16; ++v)
-      cp_async16(stg + (v * WK + wt) * 4, static_cast<const unsigned short*>(src) + e0 + 8 * wt + VS * v);
+    for (int v = 0; v < 16; ++v) {
+      const int o = 8 * wt + VS * v;
+      cp_async16_zfill(stg + (v * WK + wt) * 4, static_cast<const unsigned short*>(src) + e0 + (o < lim ? o : 0),
+                       o < lim ? 16 : 0);
+    }
   } else {
 #pragma unroll
     for (int v = 0; v < 8; ++v)
 #pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2)
-        cp_async16(stg + ((2 * v + h2) * WK + wt) * 4, static_cast<const float*>(src) + e0 + 8 * wt + VS * v + 4 * h2);
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int o = 8 * wt + VS * v + 4 * h2;
+        cp_async16_zfill(stg + ((2 * v + h2) * WK + wt) * 4, static_cast<const float*>(src) + e0 + (o < lim ? o : 0),
+                         o < lim ? 16 : 0);
+      }
   }
   cp_async_commit();
 }
@@ -295,16 +326,21 @@ __device__ __forceinline__ void round_v(float2 (&a)[16][4]) {
 //     r9, ...) with lanes on (r1, r2, r9, r10, r11).  round B: r0 (inside the pairs), r3..r8,
 //     and for R = 14 r9 by one shuffle stage.
 // The row arrives through the staging area (prefetched while the previous row was processed);
-// the next row's prefetch (element e0_next of src_next, if src_next is not null) is issued as
-// soon as this row is in registers.
+// the next row's prefetch (element e0_next of src_next, lim_next of its elements stored, if
+// src_next is not null) is issued as soon as this row is in registers.  Elements of a row at
+// offsets >= lim are zero padding (never read).
 template <int D, int R>
-__device__ __forceinline__ void row_forward_in(const void* src, long long e0, float* dst_ws, float* xbuf, float* stg,
-                                               int wt, int worker, const void* src_next, long long e0_next) {
+__device__ __forceinline__ void row_forward_in(const void* src, long long e0, int lim, float* dst_ws, float* xbuf,
+                                               float* stg, int wt, int worker, const void* src_next, long long e0_next,
+                                               int lim_next) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   float2 a[16][4];  // [vector][r1 + 2 r2]
   if constexpr (D == DT_F32) {
 #pragma unroll
-    for (int v = 8; v < 16; ++v) IOv<D>::ld8(src, e0 + 8 * wt + VS * v, a[v]);
+    for (int v = 8; v < 16; ++v) {
+      const int o = 8 * wt + VS * v;
+      IOv<D>::ld8_lim(src, e0 + (o < lim ? o : 0), a[v], lim - o);
+    }
   }
   cp_async_wait_all();
   if constexpr (D == DT_BF16) {
@@ -327,7 +363,7 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
     }
   }
   round_v(a);
-  if (src_next != nullptr) stage_row_in<D, R>(src_next, e0_next, stg, wt);
+  if (src_next != nullptr) stage_row_in<D, R>(src_next, e0_next, stg, wt, lim_next);
   // exchange V -> P
 #pragma unroll
   for (int v = 0; v < 16; ++v)
@@ -354,9 +390,10 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, fl
 // Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all R row bits (mirror of phase 1).
 // The first half of the row's pairs arrives through the staging area; src_next (if not null) is
 // the next row, whose prefetch is issued once this row is in registers.
+// Only the row's first lim elements are stored (the rest is the cropped padding).
 template <int D, int R>
-__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, float* xbuf, float* stg,
-                                                int wt, int worker, const float* src_next) {
+__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, int lim, float* xbuf,
+                                                float* stg, int wt, int worker, const float* src_next) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   const int pbase = pbase_of(wt);
   float2 b[64];
@@ -388,7 +425,19 @@ __device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, 
     for (int i = 0; i < 4; ++i) bf_in(a[v][i]);
   round_v(a);
 #pragma unroll
-  for (int v = 0; v < 16; ++v) IOv<D>::st8(dst, e0 + 8 * wt + VS * v, a[v]);
+  for (int v = 0; v < 16; ++v) IOv<D>::st8_lim(dst, e0 + 8 * wt + VS * v, a[v], lim - (8 * wt + VS * v));
+}
+
+// Where row r of the plane group that starts at plane b0 lives in X / Y (planes of lv stored
+// elements, back to back): its first element and how many of its 2^R elements are stored.
+// Rows wholly in the padding get lim = 0 and the plane's first element (never accessed).
+template <int R, int Q>
+__device__ __forceinline__ void row_loc(long long b0, long long r, long long lv, long long* e0, int* lim) {
+  const long long b = r >> Q, start = (r & ((1ll << Q) - 1)) << R;
+  long long n = lv - start;
+  n = n < 0 ? 0 : n > (1ll << R) ? (1ll << R) : n;
+  *e0 = (b0 + b) * lv + (n > 0 ? start : 0);
+  *lim = static_cast<int>(n);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -702,14 +751,22 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
           tab[i] = expf(i < n_t ? P.gt[sep_token_of<R, Q>(i, P.cbits)] : P.gc[i - n_t]);
       }
     }
-    if (rb + worker < re) stage_row_in<D, R>(P.x, (b0 << m) + ((rb + worker) << R), stg, wt);
+    if (rb + worker < re) {
+      long long e0;
+      int lim;
+      row_loc<R, Q>(b0, rb + worker, P.lv, &e0, &lim);
+      stage_row_in<D, R>(P.x, e0, stg, wt, lim);
+    }
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
       const long long rn = r + RW::NWORKERS;
       // G is first read in phase 2; its fetch into L2 is spread over phase 1 (one bulk prefetch
       // per row, together the CTA's share of G), where HBM carries only X.
       if (!SEP && b0 == 0 && wt == 0) l2_prefetch_piece(g, 4ll << m, r - rb, re - rb);
-      row_forward_in<D, R>(P.x, (b0 << m) + (r << R), ws + (r << R), xbuf, stg, wt, worker,
-                           rn < re ? P.x : nullptr, (b0 << m) + (rn << R));
+      long long e0, e0n;
+      int lim, limn;
+      row_loc<R, Q>(b0, r, P.lv, &e0, &lim);
+      row_loc<R, Q>(b0, rn, P.lv, &e0n, &limn);
+      row_forward_in<D, R>(P.x, e0, lim, ws + (r << R), xbuf, stg, wt, worker, rn < re ? P.x : nullptr, e0n, limn);
     }
     if (!gsync()) break;
     // phase 2: column bits, gain, column bits
@@ -731,8 +788,10 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     if (rb + worker < re) stage_row_out<R>(ws + ((rb + worker) << R), stg, wt);
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
       const long long rn = r + RW::NWORKERS;
-      row_forward_out<D, R>(ws + (r << R), P.y, (b0 << m) + (r << R), xbuf, stg, wt, worker,
-                            rn < re ? ws + (rn << R) : nullptr);
+      long long e0;
+      int lim;
+      row_loc<R, Q>(b0, r, P.lv, &e0, &lim);
+      row_forward_out<D, R>(ws + (r << R), P.y, e0, lim, xbuf, stg, wt, worker, rn < re ? ws + (rn << R) : nullptr);
     }
     if (b0 + P.gp < P.B && !gsync()) break;
   }

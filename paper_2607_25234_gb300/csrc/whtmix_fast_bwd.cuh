@@ -177,15 +177,23 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
     {
       const long long ub = 2 * rows * blockIdx.x / gridDim.x, ue = 2 * rows * (blockIdx.x + 1) / gridDim.x;
       auto src_of = [&](long long u) -> const void* { return u < rows ? P.x : P.dy; };
-      auto e0_of = [&](long long u) { return (b0 << m) + ((u < rows ? u : u - rows) << R); };
-      if (ub + worker < ue) stage_row_in<D, R>(src_of(ub + worker), e0_of(ub + worker), stg, wt);
+      if (ub + worker < ue) {
+        long long e0;
+        int lim;
+        const long long u = ub + worker;
+        row_loc<R, Q>(b0, u < rows ? u : u - rows, P.lv, &e0, &lim);
+        stage_row_in<D, R>(src_of(u), e0, stg, wt, lim);
+      }
       for (long long u = ub + worker; u < ue; u += RW::NWORKERS) {
         const long long un = u + RW::NWORKERS;
         // G is first read in phase 2: its fetch into L2 is spread over the first group's rows
         if (b0 == 0 && wt == 0) l2_prefetch_piece(g, 4ll << m, u - ub, ue - ub);
         float* dst = u < rows ? wsx + (u << R) : wsd + ((u - rows) << R);
-        row_forward_in<D, R>(src_of(u), e0_of(u), dst, xbuf, stg, wt, worker, un < ue ? src_of(un) : nullptr,
-                             e0_of(un));
+        long long e0, e0n;
+        int lim, limn;
+        row_loc<R, Q>(b0, u < rows ? u : u - rows, P.lv, &e0, &lim);
+        row_loc<R, Q>(b0, un < rows ? un : un - rows, P.lv, &e0n, &limn);
+        row_forward_in<D, R>(src_of(u), e0, lim, dst, xbuf, stg, wt, worker, un < ue ? src_of(un) : nullptr, e0n, limn);
       }
     }
     if (!gsync()) break;
@@ -203,8 +211,10 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
       if (rb + worker < re) stage_row_out<R>(wsd + ((rb + worker) << R), stg, wt);
       for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
         const long long rn = r + RW::NWORKERS;
-        row_forward_out<D, R>(wsd + (r << R), P.dx, (b0 << m) + (r << R), xbuf, stg, wt, worker,
-                              rn < re ? wsd + (rn << R) : nullptr);
+        long long e0;
+        int lim;
+        row_loc<R, Q>(b0, r, P.lv, &e0, &lim);
+        row_forward_out<D, R>(wsd + (r << R), P.dx, e0, lim, xbuf, stg, wt, worker, rn < re ? wsd + (rn << R) : nullptr);
       }
       dg_reduce<R>(dg, wsx, m, nb, b0 == 0, lb, le);
     }

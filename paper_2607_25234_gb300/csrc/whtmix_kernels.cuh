@@ -62,6 +62,10 @@ struct Params {
   const float* gt;
   const float* gc;
   int cbits;
+  // elements of a plane held in x, y, dy, dx (planes stored back to back, lv each); the plane the
+  // mixer transforms is those followed by 2^m - lv zeros (the token-axis zero padding).  Only the
+  // fast kernels read it; everything else runs with lv = 2^m.
+  long long lv;
 };
 
 // ---- dtype traits: storage <-> accumulator (fp32 for F32/BF16, uint32 for I32) ----

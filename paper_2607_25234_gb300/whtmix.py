@@ -18,6 +18,7 @@ import torch
 from . import build as _build
 
 __all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_separable", "backward_separable",
+           "forward_padded", "backward_padded",
            "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
            "WHTMixSeparableFunction", "pad_tokens", "EXPORTS", "library"]
 
@@ -32,7 +33,7 @@ GAIN_DTYPE = {torch.float32: torch.float32, torch.bfloat16: torch.float32, torch
 EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmix_forward_ex",
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
            "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc", "whtmix_forward_separable",
-           "whtmix_backward_separable")
+           "whtmix_backward_separable", "whtmix_forward_padded", "whtmix_backward_padded")
 
 
 class WhtmixError(RuntimeError):
@@ -66,8 +67,10 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_status_string.restype = ctypes.c_char_p
             lib.whtmix_last_cuda_error.argtypes = []
             lib.whtmix_plan.argtypes = [i64, i64]
-            lib.whtmix_forward_separable.argtypes = [p, p, p, p, i64, i64, i64, i, p]
-            lib.whtmix_backward_separable.argtypes = [p, p, p, p, p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_forward_separable.argtypes = [p, p, p, p, i64, i64, i64, i64, i, p]
+            lib.whtmix_backward_separable.argtypes = [p, p, p, p, p, p, p, i64, i64, i64, i64, i, p]
+            lib.whtmix_forward_padded.argtypes = [p, p, p, i64, i64, i64, i64, i, p]
+            lib.whtmix_backward_padded.argtypes = [p, p, p, p, p, i64, i64, i64, i64, i, p]
             for name in EXPORTS:
                 if name != "whtmix_status_string":
                     getattr(lib, name).restype = ctypes.c_int
@@ -136,31 +139,37 @@ def backward(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torch.Tenso
 
 
 def _check_log_gains(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, *others: torch.Tensor):
+    """(B, N_valid, N, C): x holds N_valid tokens per plane, g_t has the padded length N."""
     if x.dtype not in (torch.float32, torch.bfloat16):
         raise TypeError(f"separable gains need float32 or bfloat16 inputs, got {x.dtype}")
-    B, N, C = _shape(x)
-    if g_t.dtype != torch.float32 or g_c.dtype != torch.float32:
-        raise TypeError("log gains must be float32")
-    if tuple(g_t.shape) != (N,) or tuple(g_c.shape) != (C,):
+    B, n_valid, C = _shape(x)
+    if g_t.dtype != torch.float32 or g_c.dtype != torch.float32 or g_t.dim() != 1:
+        raise TypeError("log gains must be 1D float32 tensors")
+    N = g_t.shape[0]
+    if N & (N - 1) or N < max(n_valid, 1):
+        raise ValueError(f"g_t must have a power-of-two length >= the {n_valid} tokens of x, got {N}")
+    if tuple(g_c.shape) != (C,):
         raise ValueError(f"log gains must be g_t [{N}] and g_c [{C}], got {tuple(g_t.shape)} and {tuple(g_c.shape)}")
     for t in (x, g_t, g_c) + others:
         if not t.is_cuda:
             raise ValueError("WHTMix runs on CUDA tensors only")
         if not t.is_contiguous():
             raise ValueError("tensors must be contiguous")
-    return B, N, C
+    return B, n_valid, N, C
 
 
 def forward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, out: torch.Tensor | None = None,
                       stream=None) -> torch.Tensor:
     """The forward with the paper's log-domain gains (Section III-B, Eq. 2-3):
-    G[n, c] = exp(g_t[n]) exp(g_c[c])."""
-    B, N, C = _check_log_gains(x, g_t, g_c)
+    G[n, c] = exp(g_t[n]) exp(g_c[c]).  When x has fewer tokens than g_t (not a power of two), the
+    planes are zero-padded to len(g_t) tokens inside the library and y keeps x's tokens."""
+    B, n_valid, N, C = _check_log_gains(x, g_t, g_c)
     y = torch.empty_like(x) if out is None else out
     if y.shape != x.shape or y.dtype != x.dtype:
         raise ValueError("out must match x in shape and dtype")
-    _check(library().whtmix_forward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), y.data_ptr(), B, N, C,
-                                              DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_forward_separable")
+    _check(library().whtmix_forward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), y.data_ptr(), B, n_valid,
+                                              N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
+           "whtmix_forward_separable")
     return y
 
 
@@ -168,17 +177,61 @@ def backward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, dy
                        dx: torch.Tensor | None = None, dg_t: torch.Tensor | None = None,
                        dg_c: torch.Tensor | None = None, stream=None):
     """(dX, dg_t, dg_c) of forward_separable."""
-    B, N, C = _check_log_gains(x, g_t, g_c, dy)
+    B, n_valid, N, C = _check_log_gains(x, g_t, g_c, dy)
     if dy.shape != x.shape or dy.dtype != x.dtype:
         raise ValueError("dy must match x in shape and dtype")
     dx = torch.empty_like(dy) if dx is None else dx
     dg_t = torch.empty_like(g_t) if dg_t is None else dg_t
     dg_c = torch.empty_like(g_c) if dg_c is None else dg_c
     _check(library().whtmix_backward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), dy.data_ptr(),
-                                               dx.data_ptr(), dg_t.data_ptr(), dg_c.data_ptr(), B, N, C,
+                                               dx.data_ptr(), dg_t.data_ptr(), dg_c.data_ptr(), B, n_valid, N, C,
                                                DTYPE_CODE[x.dtype], _stream_ptr(stream)),
            "whtmix_backward_separable")
     return dx, dg_t, dg_c
+
+
+def _check_padded(x: torch.Tensor, g: torch.Tensor, *others: torch.Tensor):
+    """(B, N_valid, N, C) for a padded call: x holds N_valid tokens, g is the padded [N, C]."""
+    if x.dtype not in DTYPE_CODE:
+        raise TypeError(f"unsupported dtype {x.dtype}; expected float32, bfloat16 or int32")
+    B, n_valid, C = _shape(x)
+    if g.dtype != GAIN_DTYPE[x.dtype] or g.dim() != 2 or g.shape[1] != C:
+        raise ValueError(f"gains must be {GAIN_DTYPE[x.dtype]} [N, {C}]")
+    N = g.shape[0]
+    if N & (N - 1) or N < max(n_valid, 1):
+        raise ValueError(f"gains must have a power-of-two token count >= the {n_valid} tokens of x, got {N}")
+    for t in (x, g) + others:
+        if not t.is_cuda:
+            raise ValueError("WHTMix runs on CUDA tensors only")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    return B, n_valid, N, C
+
+
+def forward_padded(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """The forward on planes zero-padded from x's N_valid tokens to g's N (a power of two), inside the
+    library; y keeps x's N_valid tokens (Section III-B: pad before H_N, discard the padded outputs)."""
+    B, n_valid, N, C = _check_padded(x, g)
+    y = torch.empty_like(x) if out is None else out
+    if y.shape != x.shape or y.dtype != x.dtype:
+        raise ValueError("out must match x in shape and dtype")
+    _check(library().whtmix_forward_padded(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, n_valid, N, C,
+                                           DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_forward_padded")
+    return y
+
+
+def backward_padded(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torch.Tensor | None = None,
+                    dg: torch.Tensor | None = None, stream=None):
+    """(dX, dG) of forward_padded; dX keeps x's tokens, dG is the padded [N, C]."""
+    B, n_valid, N, C = _check_padded(x, g, dy)
+    if dy.shape != x.shape or dy.dtype != x.dtype:
+        raise ValueError("dy must match x in shape and dtype")
+    dx = torch.empty_like(dy) if dx is None else dx
+    dg = torch.empty_like(g) if dg is None else dg
+    _check(library().whtmix_backward_padded(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
+                                            B, n_valid, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
+           "whtmix_backward_padded")
+    return dx, dg
 
 
 def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool = False) -> int:

@@ -132,13 +132,13 @@ def test_no_device_reported_on_a_cpu_box(lib):
     assert fwd(lib) == 8
 
 
-def sfwd(lib, x=FAKE, gt=2 * FAKE, gc=2 * FAKE + 64, y=3 * FAKE, B=1, N=4, C=4, dtype=0):
-    return lib.whtmix_forward_separable(x, gt, gc, y, B, N, C, dtype, None)
+def sfwd(lib, x=FAKE, gt=2 * FAKE, gc=2 * FAKE + 64, y=3 * FAKE, B=1, N=4, C=4, dtype=0, nv=None):
+    return lib.whtmix_forward_separable(x, gt, gc, y, B, N if nv is None else nv, N, C, dtype, None)
 
 
 def sbwd(lib, x=FAKE, gt=2 * FAKE, gc=2 * FAKE + 64, dy=3 * FAKE, dx=4 * FAKE, dgt=5 * FAKE, dgc=5 * FAKE + 64,
-         B=1, N=4, C=4, dtype=0):
-    return lib.whtmix_backward_separable(x, gt, gc, dy, dx, dgt, dgc, B, N, C, dtype, None)
+         B=1, N=4, C=4, dtype=0, nv=None):
+    return lib.whtmix_backward_separable(x, gt, gc, dy, dx, dgt, dgc, B, N if nv is None else nv, N, C, dtype, None)
 
 
 def test_separable_rejects_invalid_arguments_before_any_device_work(lib):
@@ -161,3 +161,25 @@ def test_separable_rejects_invalid_arguments_before_any_device_work(lib):
     assert sfwd(lib, gt=2 * FAKE + 4, y=FAKE) in (0, 6, 8)
     assert sbwd(lib, dx=3 * FAKE) in (0, 6, 8)
     assert sfwd(lib, B=0) == 0
+
+
+def pfwd(lib, x=FAKE, g=2 * FAKE, y=3 * FAKE, B=1, nv=3, N=4, C=4, dtype=0):
+    return lib.whtmix_forward_padded(x, g, y, B, nv, N, C, dtype, None)
+
+
+def pbwd(lib, x=FAKE, g=2 * FAKE, dy=3 * FAKE, dx=4 * FAKE, dg=5 * FAKE, B=1, nv=3, N=4, C=4, dtype=0):
+    return lib.whtmix_backward_padded(x, g, dy, dx, dg, B, nv, N, C, dtype, None)
+
+
+def test_padded_rejects_invalid_arguments_before_any_device_work(lib):
+    assert pfwd(lib, nv=5) == 1                       # more stored tokens than the padded plane
+    assert pfwd(lib, nv=-1) == 1
+    assert pfwd(lib, N=6) == 2                        # the padded length must be a power of two
+    assert pfwd(lib, x=None) == 1
+    assert pbwd(lib, dg=None) == 1
+    assert pfwd(lib, y=FAKE + 16) == 5                # 3 x 4 f32 tokens = 48 bytes: overlaps x
+    assert pfwd(lib, y=FAKE + 48) in (0, 6, 8)        # right after x's stored tokens: no overlap
+    assert pbwd(lib, dg=FAKE + 32) == 5
+    assert pfwd(lib, nv=0) == 0 and pfwd(lib, B=0) == 0   # nothing stored: nothing to do
+    assert sfwd(lib, nv=5) == 1
+    assert sfwd(lib, nv=0) == 0
