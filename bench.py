@@ -49,7 +49,8 @@ def kernel_name(w) -> str:
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 14 if m == 23 else 13
         sep = ", separable gains" if w.gains == "separable" else ""
-        return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}>"
+        pad = ", in-kernel token padding" if w.padded_io else ""
+        return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}{pad}>"
     return "k_forward_s" if m <= 13 else "k_forward_m"
 
 
@@ -236,6 +237,9 @@ def ours(args, w):
     l2 = getattr(props, "L2_cache_size", 0) or 132 * 2**20
 
     d = inputs.workload_inputs(w, seed=rank)
+    nv = w.n_valid if w.padded_io else w.N  # tokens stored per plane in X and Y
+    if w.padded_io:
+        d["x"] = np.ascontiguousarray(d["x"][:, :nv])
     tdt = {"f32": torch.float32, "bf16": torch.bfloat16, "i32": torch.int32}[w.dtype]
     x_host = torch.from_numpy(d["x"].view(np.int16) if w.dtype == "bf16" else d["x"])
     if w.dtype == "bf16":
@@ -270,12 +274,15 @@ def ours(args, w):
     fwd = lib.whtmix_forward
     bwd = lib.whtmix_backward
     fwd_sep = lib.whtmix_forward_separable
+    fwd_pad = lib.whtmix_forward_padded
     launches_per_step = 2 if w.backward else 1
 
     def step(i):
         a = args_c[i % nsets]
         if sep:
-            rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, w.N, w.N, w.C, code, sp)
+            rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, nv, w.N, w.C, code, sp)
+        elif w.padded_io:
+            rc = fwd_pad(a[0], a[1], a[2], w.B, nv, w.N, w.C, code, sp)
         else:
             rc = fwd(a[0], a[1], a[2], w.B, w.N, w.C, code, sp)
         if rc != 0:
@@ -360,6 +367,8 @@ def ours(args, w):
                 dst.copy_(src, non_blocking=True)
             if sep:
                 whtmix.forward_separable(xd, gd[:w.N], gd[w.N:], out=yd)
+            elif w.padded_io:
+                whtmix.forward_padded(xd, gd, out=yd)
             else:
                 whtmix.forward(xd, gd, out=yd)
             if w.backward:
@@ -399,7 +408,8 @@ def ours(args, w):
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
-                       "f32" if w.dtype != "i32" else "i32", "gains": w.gains, "parallelism": f"replicas{world}",
+                       "f32" if w.dtype != "i32" else "i32", "gains": w.gains, "stored_tokens": nv,
+                       "parallelism": f"replicas{world}",
                        "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / 2**20:.0f} MiB, "
                              f"{nsets * set_bytes / l2:.1f}x L2)"},
             "hbm_gbs": achieved, "pct_of_measured_peak": 100.0 * achieved / peak,

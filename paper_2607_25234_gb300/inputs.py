@@ -92,6 +92,7 @@ class Workload:
     n_valid: int | None = None  # rows >= n_valid of X (and dY) are zero: token-axis zero padding
     description: str = ""
     gains: str = "full"   # "full": G [N, C]; "separable": log gains g_t [N], g_c [C] (Eq. 2-3)
+    padded_io: bool = False  # X, Y hold only the n_valid stored tokens; the library pads to N
 
     @property
     def L(self) -> int:
@@ -102,7 +103,7 @@ class Workload:
         backward call, which reads X, dY and G and writes dX and dG."""
         bwd = self.backward if backward is None else backward
         es = 2 if self.dtype == "bf16" else 4
-        plane = self.B * self.L * es
+        plane = self.B * (self.n_valid if self.padded_io else self.N) * self.C * es
         g = self.L * 4 if self.gains == "full" else (self.N + self.C) * 4
         fwd = 2 * plane + g
         if not bwd:
@@ -129,6 +130,14 @@ WORKLOADS = {
     "fullimage_separable_1x65536x128_bf16": Workload("fullimage_separable_1x65536x128_bf16", 1, 65536, 128, "bf16",
                                                      n_valid=2 * 135 * 240, gains="separable",
                                                      description="full-image shape, separable log gains, forward"),
+    # the two 135x240 maps stored as their 64800 tokens, padded to 65536 inside the library
+    "fullimage_padded_1x64800x128_bf16": Workload("fullimage_padded_1x64800x128_bf16", 1, 65536, 128, "bf16",
+                                                  n_valid=2 * 135 * 240, padded_io=True,
+                                                  description="64800 stored tokens, padded in the library, forward"),
+    # the paper's mixer as trained: separable log gains and in-library padding
+    "fullimage_paper_1x64800x128_bf16": Workload("fullimage_paper_1x64800x128_bf16", 1, 65536, 128, "bf16",
+                                                 n_valid=2 * 135 * 240, padded_io=True, gains="separable",
+                                                 description="64800 stored tokens, separable log gains, forward"),
 }
 WORKLOAD_ORDER = list(WORKLOADS)
 
