@@ -55,9 +55,9 @@ def test_plan_and_workspace_sizes(lib):
     import torch
     assert ws(1, 256, 32, torch.float32) == 256
     assert ws(1, 65536, 128, torch.bfloat16) == 256 + (1 << 23) * 4
-    # training step [16, 8192, 256]: forward groups of 4 planes, backward groups of 2 (two buffers)
-    assert ws(16, 8192, 256, torch.bfloat16) == 256 + 4 * (1 << 21) * 4
-    assert ws(16, 8192, 256, torch.bfloat16, backward=True) == 256 + 2 * 2 * (1 << 21) * 4
+    # training step [16, 8192, 256]: forward groups of 8 planes, backward groups of 4 (two buffers)
+    assert ws(16, 8192, 256, torch.bfloat16) == 256 + 8 * (1 << 21) * 4
+    assert ws(16, 8192, 256, torch.bfloat16, backward=True) == 256 + 4 * 2 * (1 << 21) * 4
     assert ws(0, 4, 4, torch.float32, backward=True) == 256 + 16 * 4
 
 

@@ -154,7 +154,7 @@ def test_largest_plane_2_pow_26_bf16():
 
 
 def test_many_groups_forward_and_backward_f32():
-    # 2^20 elements per plane: forward groups of 8 planes, backward groups of 4
+    # 2^20 elements per plane: forward groups of 16 planes, backward groups of 8
     run_forward(20, 4096, 256, "f32", seed=4)
     run_backward(10, 4096, 256, "f32", seed=5)
 
