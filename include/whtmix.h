@@ -167,6 +167,23 @@ WHTMIX_API int whtmix_backward_separable(const void *x, const float *g_t, const 
                                          float *dg_t, float *dg_c, int64_t B, int64_t N_valid, int64_t N, int64_t C,
                                          int dtype, void *stream);
 
+/* Token-wise channel projection on the tensor cores: z[t, :] = x[t, :] w^T for T tokens of C
+ * channels, x [T, C] bf16, w [C, C] bf16 stored (out, in) like a linear layer's weight, z [T, C]
+ * in out_dtype (WHTMIX_BF16, rounded to nearest even, or WHTMIX_F32); fp32 accumulation.  These
+ * are the block's W_in and W_out (Section III-B, Eq. 1 and Eq. 4).  C must be 64, 128 or 256
+ * (WHTMIX_ERR_BAD_SHAPE otherwise).  z may be x itself for bf16 output; no other overlap.  16-byte
+ * aligned device pointers; T = 0 is a no-op. */
+WHTMIX_API int whtmix_project(const void *x, const void *w, void *z, int64_t T, int64_t C, int out_dtype,
+                              void *stream);
+
+/* The whole mixer block of Section III-B, Eq. 1-4, forward: Z = X W_in^T, M = the mixer of Z with
+ * gains G (as whtmix_forward), Y = M W_out^T, per token row; x, y [B, N, C] bf16, w_in, w_out
+ * [C, C] bf16 (out, in), gains [N, C] fp32.  Z and M are rounded to bf16 between the steps (the
+ * block's activations), arithmetic is fp32.  dtype must be WHTMIX_BF16; C 64, 128 or 256.  y may be
+ * x itself.  Three launches on `stream` (projection, mixer, projection), each in place in y. */
+WHTMIX_API int whtmix_block_forward(const void *x, const void *w_in, const void *gains, const void *w_out, void *y,
+                                    int64_t B, int64_t N, int64_t C, int dtype, void *stream);
+
 /* Synchronises `stream` and reports device-side failures of the calls enqueued on it since the
  * previous whtmix_sync: WHTMIX_ERR_TIMEOUT if a bounded device-wide wait gave up (the library
  * then resets that workspace's barrier), WHTMIX_ERR_CUDA if the synchronisation itself failed,

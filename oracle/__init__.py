@@ -157,3 +157,12 @@ def backward_separable(x: np.ndarray, g_t: np.ndarray, g_c: np.ndarray, dy: np.n
     G = separable_gains(g_t, g_c)
     dx, dG = backward(np.asarray(x, dtype=np.float64), G, np.asarray(dy, dtype=np.float64))
     return dx, (dG * G).sum(axis=1), (dG * G).sum(axis=0)
+
+
+def block_forward(x: np.ndarray, w_in: np.ndarray, g: np.ndarray, w_out: np.ndarray) -> np.ndarray:
+    """The whole mixer block of Section III-B, Eq. 1-4, in float64: Z = X W_in^T per token (the input
+    projection), the 2D WHT mixer of Z with gains G, then the output projection M W_out^T.  The
+    weights are stored (out, in), as a linear layer's."""
+    x = np.asarray(x, dtype=np.float64)
+    z = x @ np.asarray(w_in, dtype=np.float64).T
+    return forward(z, np.asarray(g, dtype=np.float64)) @ np.asarray(w_out, dtype=np.float64).T

@@ -15,6 +15,14 @@
 #include "whtmix_fast_launch.cuh"
 #include "whtmix_kernels.cuh"
 
+namespace whtmix {
+namespace proj {
+// whtmix_proj.cu: Z = X W^T on the tensor cores (C = 64, 128, 256; bf16 in, bf16 or fp32 out)
+cudaError_t project(const void* x, const void* w, void* z, long long T, int C, bool out_f32, unsigned int* err, int sms,
+                    cudaStream_t s);
+}  // namespace proj
+}  // namespace whtmix
+
 using namespace whtmix;
 
 namespace {
@@ -629,6 +637,56 @@ int whtmix_backward_separable(const void* x, const float* g_t, const float* g_c,
                               void* stream) {
   return run(separable_call(true, x, g_t, g_c, dy, dx, dg_t, dg_c, B, N_valid, N, C, dtype), nullptr, 0, false,
              stream);
+}
+
+int whtmix_project(const void* x, const void* w, void* z, int64_t T, int64_t C, int out_dtype, void* stream_v) {
+  if (T < 0 || C < 1) return WHTMIX_ERR_INVALID_ARG;
+  if (C != 64 && C != 128 && C != 256) return WHTMIX_ERR_BAD_SHAPE;
+  if (out_dtype != WHTMIX_F32 && out_dtype != WHTMIX_BF16) return WHTMIX_ERR_BAD_DTYPE;
+  if (T == 0) return WHTMIX_OK;
+  if (!x || !w || !z) return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(w) || !aligned16(z)) return WHTMIX_ERR_MISALIGNED;
+  const size_t xb = static_cast<size_t>(T) * C * 2, wb = static_cast<size_t>(C) * C * 2;
+  const size_t zb = static_cast<size_t>(T) * C * (out_dtype == WHTMIX_F32 ? 4 : 2);
+  // z may be x itself (bf16 out: each tile is read whole before it is written), nothing else
+  if (!(z == x && out_dtype == WHTMIX_BF16) && overlap(z, zb, x, xb)) return WHTMIX_ERR_ALIAS;
+  if (overlap(z, zb, w, wb)) return WHTMIX_ERR_ALIAS;
+  int dev = 0, sms = 0;
+  int rc = device_check(&dev, &sms);
+  if (rc != WHTMIX_OK) return rc;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  void* ws = nullptr;
+  rc = cached_workspace(dev, stream, HEADER_BYTES, &ws);
+  if (rc != WHTMIX_OK) return rc;
+  const cudaError_t e = proj::project(x, w, z, T, static_cast<int>(C), out_dtype == WHTMIX_F32,
+                                      &static_cast<GridBarrier*>(ws)->err, sms, stream);
+  return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+}
+
+int whtmix_block_forward(const void* x, const void* w_in, const void* gains, const void* w_out, void* y, int64_t B,
+                         int64_t N, int64_t C, int dtype, void* stream) {
+  int m = 0;
+  int rc = check_shape(B, N, C, dtype, &m);
+  if (rc != WHTMIX_OK) return rc;
+  if (dtype != WHTMIX_BF16) return WHTMIX_ERR_BAD_DTYPE;
+  if (C != 64 && C != 128 && C != 256) return WHTMIX_ERR_BAD_SHAPE;
+  if (B == 0) return WHTMIX_OK;
+  if (!x || !w_in || !gains || !w_out || !y) return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(w_in) || !aligned16(gains) || !aligned16(w_out) || !aligned16(y))
+    return WHTMIX_ERR_MISALIGNED;
+  const size_t plane_bytes = static_cast<size_t>(B) * N * C * 2, wb = static_cast<size_t>(C) * C * 2;
+  const size_t g_bytes = static_cast<size_t>(N) * C * 4;
+  // y is written three times (projection, mixer, projection), so it may not hold any input except x
+  if (y != x && overlap(y, plane_bytes, x, plane_bytes)) return WHTMIX_ERR_ALIAS;
+  if (overlap(y, plane_bytes, w_in, wb) || overlap(y, plane_bytes, w_out, wb) || overlap(y, plane_bytes, gains, g_bytes))
+    return WHTMIX_ERR_ALIAS;
+  const long long T = B * N;
+  // Eq. 1: Z = X W_in^T, into y; Eq. 2-3: the mixer, in place; Eq. 4: Y = M W_out^T, in place
+  rc = whtmix_project(x, w_in, y, T, C, WHTMIX_BF16, stream);
+  if (rc != WHTMIX_OK) return rc;
+  rc = run(full_call(false, y, gains, nullptr, y, nullptr, B, N, N, C, dtype), nullptr, 0, false, stream);
+  if (rc != WHTMIX_OK) return rc;
+  return whtmix_project(y, w_out, y, T, C, WHTMIX_BF16, stream);
 }
 
 int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype, int backward, size_t* out_bytes) {

@@ -1,0 +1,204 @@
+// whtmix_proj.cu -- token-wise channel projection on the 5th-generation tensor cores:
+//   Z[t, :] = X[t, :] W^T        X [T, C] bf16, W [C, C] bf16 (out, in), Z [T, C] bf16 or fp32
+// the W_in and W_out projections around the mixer (Section III-B, Eq. 1 and Eq. 4).
+//
+// One persistent CTA per SM (the shared-memory request leaves room for one), 128 threads: tiles
+// of 128 tokens.  W is staged in shared memory once per CTA; each tile of X is staged next to it;
+// one thread issues C/16 tcgen05.mma (kind::f16, bf16 x bf16 -> fp32, M = 128, N = C, K = 16) with
+// the accumulator in TMEM (lane = token of the tile, column = output channel) and commits them to
+// an mbarrier; every thread then reads its token's row of the accumulator with tcgen05.ld and
+// stores it.  Both operands are K-major (X rows are tokens with their channels contiguous, W rows
+// are output channels with their input channels contiguous), laid out in shared memory as the
+// tensor core's no-swizzle canonical form: 8-row x 16-byte core matrices, the K-adjacent core
+// matrix 128 bytes on, the next group of 8 rows (C / 8) x 128 bytes on.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "whtmix_kernels.cuh"
+
+namespace whtmix {
+namespace proj {
+
+constexpr int THREADS = 128;   // one thread per TMEM lane = per token of a tile
+constexpr int TILE_T = 128;    // tokens per tile (the MMA's M)
+constexpr size_t SMEM_MIN = 120 * 1024;  // more than half an SM: one CTA per SM, so TMEM allocation never waits
+constexpr long long WAIT_LIMIT = 1ll << 26;  // polls of an mbarrier before giving up
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
+
+// Shared-memory matrix descriptor, no swizzle: start address, leading-dimension byte offset (the
+// K-adjacent core matrix), stride byte offset (the next 8-row group), descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  return static_cast<uint64_t>((addr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(lbo >> 4) << 16) |
+         (static_cast<uint64_t>(sbo >> 4) << 32) | (1ull << 46);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both K-major, N, M.
+__host__ __device__ constexpr uint32_t instr_desc(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// Byte offset of element (row r, k) of a K-major operand with K columns in the canonical layout.
+__device__ __forceinline__ uint32_t core_off(int r, int k, int K) {
+  return static_cast<uint32_t>(((r >> 3) * (K >> 3) + (k >> 3)) * 128 + (r & 7) * 16 + (k & 7) * 2);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+// Bounded wait for phase `parity` of an mbarrier; false if it did not complete.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  const uint32_t a = smem_u32(bar);
+  for (long long i = 0; i < WAIT_LIMIT; ++i) {
+    uint32_t done;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(done) : "r"(a), "r"(parity) : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols) : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+               ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate) : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t ta, float (&r)[16]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+               : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]), "=f"(r[6]), "=f"(r[7]),
+                 "=f"(r[8]), "=f"(r[9]), "=f"(r[10]), "=f"(r[11]), "=f"(r[12]), "=f"(r[13]), "=f"(r[14]), "=f"(r[15])
+               : "r"(ta) : "memory");
+}
+
+// C in {64, 128, 256}; OUT_F32: fp32 output (else bf16, round to nearest even).
+template <int C, bool OUT_F32>
+__global__ void __launch_bounds__(THREADS, 1) k_proj(const __nv_bfloat16* x, const __nv_bfloat16* __restrict__ w,
+                                                     void* z, long long T, unsigned int* err) {  // z may be x
+  static_assert(C == 64 || C == 128 || C == 256, "channels");
+  extern __shared__ __align__(1024) unsigned char smem[];
+  __shared__ uint64_t mbar;
+  __shared__ uint32_t tmem_slot;
+  unsigned char* sw = smem;                     // W: C x C bf16, canonical layout
+  unsigned char* sx = smem + C * C * 2;         // X tile: 128 x C bf16, canonical layout
+  const int tid = threadIdx.x;
+  // W once per CTA
+  for (int i = tid; i < C * C / 8; i += THREADS) {
+    const int r = i / (C / 8), k = (i % (C / 8)) * 8;
+    *reinterpret_cast<uint4*>(sw + core_off(r, k, C)) = *reinterpret_cast<const uint4*>(w + static_cast<long long>(r) * C + k);
+  }
+  if (tid < 32) tmem_alloc(&tmem_slot, C);
+  if (tid == 0) {
+    mbar_init(&mbar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = tmem_slot;
+  const uint32_t idesc = instr_desc(TILE_T, C);
+  const uint32_t lane_base = static_cast<uint32_t>(32 * (tid >> 5)) << 16;
+  const long long ntiles = (T + TILE_T - 1) / TILE_T;
+  uint32_t parity = 0;
+  bool ok = true;
+  for (long long tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+    const long long t0 = tile * TILE_T;
+    // X tile; tokens past T are zero
+    for (int i = tid; i < TILE_T * C / 8; i += THREADS) {
+      const int r = i / (C / 8), k = (i % (C / 8)) * 8;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (t0 + r < T) v = *reinterpret_cast<const uint4*>(x + (t0 + r) * C + k);
+      *reinterpret_cast<uint4*>(sx + core_off(r, k, C)) = v;
+    }
+    // generic-proxy shared-memory writes -> visible to the tensor core (async proxy)
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncthreads();
+    if (tid == 0) {
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const uint32_t ax = smem_u32(sx), aw = smem_u32(sw);
+#pragma unroll
+      for (int ks = 0; ks < C / 16; ++ks)  // K steps of 16: two core matrices along K
+        mma_bf16(tmem, smem_desc(ax + ks * 256, 128, (C / 8) * 128), smem_desc(aw + ks * 256, 128, (C / 8) * 128), idesc,
+                 ks > 0 ? 1u : 0u);
+      mma_commit(&mbar);
+    }
+    // every thread waits; the CTA goes on only if all saw the MMAs complete (a uniform decision,
+    // so that no thread is left at a later barrier)
+    ok = __syncthreads_and(mbar_wait(&mbar, parity) ? 1 : 0) != 0;
+    if (!ok) {
+      if (tid == 0) atomicOr(err, 1u);
+      break;
+    }
+    parity ^= 1u;
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    // row tid of the tile: C accumulator columns of TMEM lane tid
+    const long long t = t0 + tid;
+#pragma unroll
+    for (int c0 = 0; c0 < C; c0 += 16) {
+      float v[16];
+      tmem_ld16(tmem + lane_base + c0, v);
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      if (t < T) {
+        if constexpr (OUT_F32) {
+          float4* o = reinterpret_cast<float4*>(static_cast<float*>(z) + t * C + c0);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        } else {
+          uint32_t h[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            __nv_bfloat162 b = __floats2bfloat162_rn(v[2 * q], v[2 * q + 1]);
+            h[q] = *reinterpret_cast<uint32_t*>(&b);
+          }
+          uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(z) + t * C + c0);
+          o[0] = make_uint4(h[0], h[1], h[2], h[3]);
+          o[1] = make_uint4(h[4], h[5], h[6], h[7]);
+        }
+      }
+    }
+    // every thread's TMEM reads are done before the next tile's MMAs overwrite the accumulator,
+    // and the MMAs (complete, per the mbarrier) no longer read the X tile
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+  }
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (tid < 32) tmem_dealloc(tmem, C);
+}
+
+template <int C, bool OUT_F32>
+cudaError_t launch_c(const void* x, const void* w, void* z, long long T, unsigned int* err, int sms, cudaStream_t s) {
+  const size_t need = static_cast<size_t>(C) * C * 2 + static_cast<size_t>(TILE_T) * C * 2;
+  const size_t smem = need > SMEM_MIN ? need : SMEM_MIN;
+  auto k = k_proj<C, OUT_F32>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const long long ntiles = (T + TILE_T - 1) / TILE_T;
+  const unsigned grid = static_cast<unsigned>(ntiles < sms ? ntiles : sms);
+  k<<<grid, THREADS, smem, s>>>(static_cast<const __nv_bfloat16*>(x), static_cast<const __nv_bfloat16*>(w), z, T, err);
+  return cudaGetLastError();
+}
+
+// Z = X W^T for T tokens of C channels (C = 64, 128 or 256); err: device word set on a timeout.
+cudaError_t project(const void* x, const void* w, void* z, long long T, int C, bool out_f32, unsigned int* err, int sms,
+                    cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  switch (C) {
+    case 64: return out_f32 ? launch_c<64, true>(x, w, z, T, err, sms, s) : launch_c<64, false>(x, w, z, T, err, sms, s);
+    case 128: return out_f32 ? launch_c<128, true>(x, w, z, T, err, sms, s) : launch_c<128, false>(x, w, z, T, err, sms, s);
+    case 256: return out_f32 ? launch_c<256, true>(x, w, z, T, err, sms, s) : launch_c<256, false>(x, w, z, T, err, sms, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace proj
+}  // namespace whtmix

@@ -18,7 +18,7 @@ import torch
 from . import build as _build
 
 __all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_separable", "backward_separable",
-           "forward_padded", "backward_padded",
+           "forward_padded", "backward_padded", "project", "block_forward",
            "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
            "WHTMixSeparableFunction", "pad_tokens", "EXPORTS", "library"]
 
@@ -33,7 +33,8 @@ GAIN_DTYPE = {torch.float32: torch.float32, torch.bfloat16: torch.float32, torch
 EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmix_forward_ex",
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
            "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc", "whtmix_forward_separable",
-           "whtmix_backward_separable", "whtmix_forward_padded", "whtmix_backward_padded")
+           "whtmix_backward_separable", "whtmix_forward_padded", "whtmix_backward_padded", "whtmix_project",
+           "whtmix_block_forward")
 
 
 class WhtmixError(RuntimeError):
@@ -70,6 +71,8 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_forward_separable.argtypes = [p, p, p, p, i64, i64, i64, i64, i, p]
             lib.whtmix_backward_separable.argtypes = [p, p, p, p, p, p, p, i64, i64, i64, i64, i, p]
             lib.whtmix_forward_padded.argtypes = [p, p, p, i64, i64, i64, i64, i, p]
+            lib.whtmix_project.argtypes = [p, p, p, i64, i64, i, p]
+            lib.whtmix_block_forward.argtypes = [p, p, p, p, p, i64, i64, i64, i, p]
             lib.whtmix_backward_padded.argtypes = [p, p, p, p, p, i64, i64, i64, i64, i, p]
             for name in EXPORTS:
                 if name != "whtmix_status_string":
@@ -232,6 +235,37 @@ def backward_padded(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torc
                                             B, n_valid, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
            "whtmix_backward_padded")
     return dx, dg
+
+
+def project(x: torch.Tensor, w: torch.Tensor, out_dtype: torch.dtype = torch.bfloat16,
+            out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """z = x w^T per token on the tensor cores (x [..., C] bf16, w [C, C] bf16 as (out, in))."""
+    if x.dtype != torch.bfloat16 or w.dtype != torch.bfloat16:
+        raise TypeError("project takes bfloat16 x and w")
+    C = x.shape[-1]
+    if tuple(w.shape) != (C, C):
+        raise ValueError(f"w must be [{C}, {C}]")
+    for t in (x, w):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("x and w must be contiguous CUDA tensors")
+    z = torch.empty(x.shape, dtype=out_dtype, device=x.device) if out is None else out
+    _check(library().whtmix_project(x.data_ptr(), w.data_ptr(), z.data_ptr(), x.numel() // C, C,
+                                    DTYPE_CODE[out_dtype], _stream_ptr(stream)), "whtmix_project")
+    return z
+
+
+def block_forward(x: torch.Tensor, w_in: torch.Tensor, g: torch.Tensor, w_out: torch.Tensor,
+                  out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """The mixer block of Section III-B, Eq. 1-4: Y = mix(X W_in^T) W_out^T (bf16)."""
+    B, N, C = _check_tensors(x, g)
+    for t in (w_in, w_out):
+        if t.dtype != torch.bfloat16 or tuple(t.shape) != (C, C) or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"w_in and w_out must be contiguous bfloat16 CUDA tensors [{C}, {C}]")
+    y = torch.empty_like(x) if out is None else out
+    _check(library().whtmix_block_forward(x.data_ptr(), w_in.data_ptr(), g.data_ptr(), w_out.data_ptr(),
+                                          y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
+           "whtmix_block_forward")
+    return y
 
 
 def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool = False) -> int:

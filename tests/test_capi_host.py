@@ -183,3 +183,21 @@ def test_padded_rejects_invalid_arguments_before_any_device_work(lib):
     assert pfwd(lib, nv=0) == 0 and pfwd(lib, B=0) == 0   # nothing stored: nothing to do
     assert sfwd(lib, nv=5) == 1
     assert sfwd(lib, nv=0) == 0
+
+
+def test_project_and_block_reject_invalid_arguments_before_any_device_work(lib):
+    P = lib.whtmix_project
+    assert P(FAKE, 2 * FAKE, 3 * FAKE, 1, 96, 1, None) == 2        # C must be 64, 128 or 256
+    assert P(FAKE, 2 * FAKE, 3 * FAKE, 1, 64, 2, None) == 3        # output fp32 or bf16
+    assert P(FAKE, 2 * FAKE, 3 * FAKE, -1, 64, 1, None) == 1
+    assert P(None, 2 * FAKE, 3 * FAKE, 1, 64, 1, None) == 1
+    assert P(FAKE + 8, 2 * FAKE, 3 * FAKE, 1, 64, 1, None) == 4
+    assert P(FAKE, 2 * FAKE, FAKE + 16, 4, 64, 1, None) == 5       # partial overlap with x
+    assert P(FAKE, 2 * FAKE, 2 * FAKE, 4, 64, 1, None) == 5        # output over w
+    assert P(FAKE, 2 * FAKE, FAKE, 4, 64, 0, None) == 5            # in place only with bf16 output
+    assert P(FAKE, 2 * FAKE, 3 * FAKE, 0, 64, 1, None) == 0        # no tokens
+    Bk = lib.whtmix_block_forward
+    assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 5 * FAKE, 1, 4, 64, 0, None) == 3   # bf16 only
+    assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 5 * FAKE, 1, 4, 32, 1, None) == 2   # C 64, 128 or 256
+    assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 2 * FAKE, 1, 4, 64, 1, None) == 5   # y over w_in
+    assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 5 * FAKE, 0, 4, 64, 1, None) == 0

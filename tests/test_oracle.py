@@ -210,6 +210,23 @@ def test_separable_backward_finite_differences(B, N, C):
     assert abs(dgc.sum() - total) <= 1e-10 * max(1.0, abs(total))
 
 
+@pytest.mark.parametrize("B,N,C", [(1, 8, 4), (2, 16, 8), (1, 4, 16)])
+def test_block_forward_dense_and_special_cases(B, N, C):
+    # dense: H_N (G (.) H_N (X W_in^T) H_C) H_C W_out^T / (N C) with scipy Hadamard matrices
+    x = rng_normal((B, N, C), 60)
+    w_in, w_out = rng_normal((C, C), 61), rng_normal((C, C), 62)
+    g = 1.0 + 0.1 * rng_normal((N, C), 63)
+    hn = scipy.linalg.hadamard(N).astype(np.float64)
+    hc = scipy.linalg.hadamard(C).astype(np.float64)
+    want = np.stack([hn @ (g * (hn @ (xb @ w_in.T) @ hc)) @ hc @ w_out.T for xb in x]) / (N * C)
+    np.testing.assert_allclose(oracle.block_forward(x, w_in, g, w_out), want, rtol=1e-11, atol=1e-12)
+    # identity projections: the mixer alone; unit gains: the two projections alone
+    eye = np.eye(C)
+    np.testing.assert_allclose(oracle.block_forward(x, eye, g, eye), oracle.forward(x, g), rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(oracle.block_forward(x, w_in, np.ones((N, C)), w_out), x @ w_in.T @ w_out.T,
+                               rtol=1e-11, atol=1e-12)
+
+
 def test_linear_in_x_and_in_g():
     N, C = 32, 16
     x1, x2 = rng_normal((N, C), 20), rng_normal((N, C), 21)
