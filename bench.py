@@ -50,7 +50,8 @@ def kernel_name(w) -> str:
         r = 14 if m == 23 else 13
         sep = ", separable gains" if w.gains == "separable" else ""
         pad = ", in-kernel token padding" if w.padded_io else ""
-        return f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}{pad}>"
+        name = f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}{pad}>"
+        return f"k_proj<C={w.C}> + {name} + k_proj<C={w.C}>" if w.block else name
     return "k_forward_s" if m <= 13 else "k_forward_m"
 
 
@@ -151,11 +152,14 @@ def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
     g = d["g"].astype(np.float64)
     dy = inputs.as_float64(d["dy"], w.dtype) if w.backward else None
     g_t, g_c = (a.astype(np.float64) for a in inputs.make_log_gains(n_tokens, w.C, 0))
+    w_in, w_out = (inputs.as_float64(a, "bf16") for a in inputs.make_projections(w.C, 0))
     oracle.forward(x[:, :8, :], g[:8, :])  # load / compile outside the timing
     times = []
     for _ in range(reps):
         t = time.perf_counter()
-        if w.gains == "separable":
+        if w.block:
+            oracle.block_forward(x, w_in, g, w_out)
+        elif w.gains == "separable":
             oracle.forward_separable(x, g_t, g_c)
         else:
             oracle.forward(x, g)
@@ -182,7 +186,10 @@ def reference_arm(args, w):
     d = inputs.make_inputs(1, n, w.C, w.dtype, seed=0, n_valid=None if w.n_valid is None else min(w.n_valid, n))
     x = inputs.as_float64(d["x"], w.dtype)
     g = d["g"].astype(np.float64)
-    if w.gains == "separable":
+    if w.block:
+        w_in, w_out = (inputs.as_float64(a, "bf16") for a in inputs.make_projections(w.C, 0))
+        run = lambda: oracle.block_forward(x, w_in, g, w_out)
+    elif w.gains == "separable":
         g_t, g_c = (a.astype(np.float64) for a in inputs.make_log_gains(n, w.C, 0))
         run = lambda: oracle.forward_separable(x, g_t, g_c)
     else:
@@ -195,7 +202,8 @@ def reference_arm(args, w):
     el = time.perf_counter() - t0
     value = args.steps * n / el
     sample = f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s)"
-    line = {"impl": "reference", "metric": "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s",
+    metric = "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
+    line = {"impl": "reference", "metric": metric, "value": value, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * el / max(args.steps, 1), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -275,11 +283,17 @@ def ours(args, w):
     bwd = lib.whtmix_backward
     fwd_sep = lib.whtmix_forward_separable
     fwd_pad = lib.whtmix_forward_padded
-    launches_per_step = 2 if w.backward else 1
+    fwd_block = lib.whtmix_block_forward
+    launches_per_step = 2 if w.backward else 3 if w.block else 1
+    if w.block:
+        wi = torch.from_numpy(d["w_in"].view(np.int16)).to(dev).view(torch.bfloat16)
+        wo = torch.from_numpy(d["w_out"].view(np.int16)).to(dev).view(torch.bfloat16)
 
     def step(i):
         a = args_c[i % nsets]
-        if sep:
+        if w.block:
+            rc = fwd_block(a[0], wi.data_ptr(), a[1], wo.data_ptr(), a[2], w.B, w.N, w.C, code, sp)
+        elif sep:
             rc = fwd_sep(a[0], a[1], a[1] + 4 * w.N, a[2], w.B, nv, w.N, w.C, code, sp)
         elif w.padded_io:
             rc = fwd_pad(a[0], a[1], a[2], w.B, nv, w.N, w.C, code, sp)
@@ -365,7 +379,9 @@ def ours(args, w):
         def e2e_step():
             for dst, src in h2d:
                 dst.copy_(src, non_blocking=True)
-            if sep:
+            if w.block:
+                whtmix.block_forward(xd, wi, gd, wo, out=yd)
+            elif sep:
                 whtmix.forward_separable(xd, gd[:w.N], gd[w.N:], out=yd)
             elif w.padded_io:
                 whtmix.forward_padded(xd, gd, out=yd)
@@ -404,7 +420,8 @@ def ours(args, w):
                          f"median of {len(times)} run(s): "
                          + ", ".join(f"{t:.2f}" for t in times) + " s"}
 
-    line = {"metric": "WHTMix fwd+bwd tokens/s" if w.backward else "WHTMix fwd tokens/s", "value": value, "unit": "tokens/s", "n_gpus": world,
+    metric = "WHTMix fwd+bwd tokens/s" if w.backward else "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
+    line = {"metric": metric, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":

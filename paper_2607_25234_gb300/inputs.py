@@ -6,7 +6,8 @@ no part of the mixer's arithmetic: it draws numbers and quantises them to the st
 Generator: SplitMix64 (Steele, Lea & Flood, "Fast splittable pseudorandom number generators",
 OOPSLA 2014) -> 53-bit uniforms in [0, 1) -> Box-Muller normals in float64.  Each tensor has its
 own stream: X uses ``seed``, G uses ``seed + 1`` and dY uses ``seed + 2``; the separable log
-gains g_t and g_c use ``seed + 3`` and ``seed + 4``.
+gains g_t and g_c use ``seed + 3`` and ``seed + 4``, the block's projections ``seed + 5`` and
+``seed + 6``.
 
 Stand-in data.  The paper trains and times the mixer on joint left+right stereo token sequences
 (Section III-A; N = 2 (H/8)(W/8), C = 64) and on LRA byte sequences (Section IV-D).  None of those
@@ -93,6 +94,7 @@ class Workload:
     description: str = ""
     gains: str = "full"   # "full": G [N, C]; "separable": log gains g_t [N], g_c [C] (Eq. 2-3)
     padded_io: bool = False  # X, Y hold only the n_valid stored tokens; the library pads to N
+    block: bool = False      # the whole block of Eq. 1-4: W_in projection, mixer, W_out projection
 
     @property
     def L(self) -> int:
@@ -105,6 +107,8 @@ class Workload:
         es = 2 if self.dtype == "bf16" else 4
         plane = self.B * (self.n_valid if self.padded_io else self.N) * self.C * es
         g = self.L * 4 if self.gains == "full" else (self.N + self.C) * 4
+        if self.block:
+            g += 2 * self.C * self.C * 2  # W_in and W_out, bf16
         fwd = 2 * plane + g
         if not bwd:
             return fwd
@@ -134,6 +138,10 @@ WORKLOADS = {
     "fullimage_padded_1x64800x128_bf16": Workload("fullimage_padded_1x64800x128_bf16", 1, 65536, 128, "bf16",
                                                   n_valid=2 * 135 * 240, padded_io=True,
                                                   description="64800 stored tokens, padded in the library, forward"),
+    # the whole mixer block (W_in, mixer, W_out) on the full-image shape
+    "block_fullimage_1x65536x128_bf16": Workload("block_fullimage_1x65536x128_bf16", 1, 65536, 128, "bf16",
+                                                 n_valid=2 * 135 * 240, block=True,
+                                                 description="mixer block: projection, mixer, projection"),
     # the paper's mixer as trained: separable log gains and in-library padding
     "fullimage_paper_1x64800x128_bf16": Workload("fullimage_paper_1x64800x128_bf16", 1, 65536, 128, "bf16",
                                                  n_valid=2 * 135 * 240, padded_io=True, gains="separable",
@@ -193,7 +201,16 @@ def workload_inputs(w: Workload, seed: int = 0) -> dict[str, np.ndarray]:
     d = make_inputs(w.B, w.N, w.C, w.dtype, seed, n_valid=w.n_valid, with_dy=w.backward)
     if w.gains == "separable":
         d["g_t"], d["g_c"] = make_log_gains(w.N, w.C, seed)
+    if w.block:
+        d["w_in"], d["w_out"] = make_projections(w.C, seed)
     return d
+
+
+def make_projections(C: int, seed: int = 0) -> tuple[np.ndarray, np.ndarray]:
+    """W_in, W_out [C, C] as bf16 bits, entries ~ N(0, 1/C) (unit-variance outputs)."""
+    w_in = (normal(seed + 5, C * C) / np.sqrt(C)).astype(np.float32).reshape(C, C)
+    w_out = (normal(seed + 6, C * C) / np.sqrt(C)).astype(np.float32).reshape(C, C)
+    return f32_to_bf16_bits(w_in).reshape(C, C), f32_to_bf16_bits(w_out).reshape(C, C)
 
 
 def as_float64(a: np.ndarray, dtype: str) -> np.ndarray:
