@@ -86,6 +86,24 @@ def dist_env():
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
 
 
+def max_over_ranks(value: float, world: int, device) -> float:
+    """The job's time is its slowest rank's: a MAX all-reduce over the ranks (each timed the same
+    K steps between two barriers)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.item()
+
+
+def whole_job_tokens_per_s(world: int, tokens_per_step: int, steps: int, elapsed_ms: float) -> float:
+    """Weak scaling, replicas: every rank runs the whole workload, so the job processes world times
+    the tokens of one step per step."""
+    return world * tokens_per_step * steps / (elapsed_ms / 1e3)
+
+
 class ClockSampler:
     """nvidia-smi samples (timestamped on the host) for one GPU while the bench runs."""
 
@@ -347,13 +365,9 @@ def ours(args, w):
     sampler.stop()
     clocks = sampler.summary(t_host0, t_host1)
 
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = t.item()
-
+    elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     tokens_per_step = w.B * w.N
-    value = world * tokens_per_step * K / (elapsed_ms / 1e3)
+    value = whole_job_tokens_per_s(world, tokens_per_step, K, elapsed_ms)
     kern_mean_ms = statistics.mean(kern_ms)
     ideal = w.ideal_bytes()
     peak, peak_kind = measured_peaks()
