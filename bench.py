@@ -40,12 +40,21 @@ REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_c
            0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
            0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_25234_gb300", "csrc", f) for f in
-                  ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_capi.cu")]
+                  ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_capi.cu",
+                   "whtmix_block.cuh", "whtmix_block.cu")]
+
+
+def block_fused(w) -> bool:
+    """True where whtmix_block_forward runs the whole block as one fused launch (mirrors the C ABI)."""
+    m = (w.N * w.C).bit_length() - 1
+    return w.block and w.dtype == "bf16" and w.C == 128 and 21 <= m <= 23
 
 
 def kernel_name(w) -> str:
     """The kernel one whtmix_forward call launches for this workload (mirrors the C ABI's dispatch)."""
     m = (w.N * w.C).bit_length() - 1
+    if block_fused(w):
+        return f"k_block_fast<bf16, R=14, Q={m - 14}>"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 14 if m == 23 else 13
         sep = ", separable gains" if w.gains == "separable" else ""
@@ -302,7 +311,7 @@ def ours(args, w):
     fwd_sep = lib.whtmix_forward_separable
     fwd_pad = lib.whtmix_forward_padded
     fwd_block = lib.whtmix_block_forward
-    launches_per_step = 2 if w.backward else 3 if w.block else 1
+    launches_per_step = 2 if w.backward else 3 if w.block and not block_fused(w) else 1
     if w.block:
         wi = torch.from_numpy(d["w_in"].view(np.int16)).to(dev).view(torch.bfloat16)
         wo = torch.from_numpy(d["w_out"].view(np.int16)).to(dev).view(torch.bfloat16)

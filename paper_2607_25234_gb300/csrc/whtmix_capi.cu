@@ -16,6 +16,10 @@
 #include "whtmix_kernels.cuh"
 
 namespace whtmix {
+namespace blk {
+// Fused block (whtmix_block.cu): bf16, C = 128, 2^21 <= N C <= 2^23, full gains, N_valid = N.
+cudaError_t forward_bf16(const Params& P, const void* w_in, const void* w_out, int sms, cudaStream_t stream);
+}  // namespace blk
 namespace proj {
 // whtmix_proj.cu: Z = X W^T on the tensor cores (C = 64, 128, 256; bf16 in, bf16 or fp32 out)
 cudaError_t project(const void* x, const void* w, void* z, long long T, int C, bool out_f32, unsigned int* err, int sms,
@@ -351,6 +355,9 @@ struct Call {
   float* dgc = nullptr;
   int64_t B = 0, n_valid = 0, N = 0, C = 0;
   int dtype = 0;
+  // the mixer block's projections (Eq. 1 and 4), fused into the forward; null for the mixer alone
+  const void* w_in = nullptr;
+  const void* w_out = nullptr;
 };
 
 // Workspace layout of a call: the kernel workspace (barrier header + plane group) first, then
@@ -501,6 +508,10 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
   P.cbits = cbits;
   P.lv = static_cast<long long>(lv);
   cudaError_t e = cudaSuccess;
+  if (c.w_in) {
+    e = blk::forward_bf16(P, c.w_in, c.w_out, sms, stream);
+    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+  }
   if (lay.fast_sep) {
     e = c.dtype == WHTMIX_BF16 ? fast::forward_sep_bf16(P, sms, stream) : fast::forward_sep_f32(P, sms, stream);
     return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
@@ -592,6 +603,10 @@ Call separable_call(bool backward, const void* x, const float* gt, const float* 
   return c;
 }
 
+// The fused block kernel covers 128 channels and planes of 2^21 to 2^23 elements (rows of 128
+// tokens x 128 channels, columns of 128 to 512 rows).
+bool use_fused_block(int64_t C, int m) { return C == 128 && m >= 21 && m <= 23; }
+
 }  // namespace
 
 extern "C" {
@@ -680,6 +695,13 @@ int whtmix_block_forward(const void* x, const void* w_in, const void* gains, con
   if (y != x && overlap(y, plane_bytes, x, plane_bytes)) return WHTMIX_ERR_ALIAS;
   if (overlap(y, plane_bytes, w_in, wb) || overlap(y, plane_bytes, w_out, wb) || overlap(y, plane_bytes, gains, g_bytes))
     return WHTMIX_ERR_ALIAS;
+  if (use_fused_block(C, m)) {
+    // one launch: the projections are the prologue and epilogue of the mixer's row phases
+    Call c = full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype);
+    c.w_in = w_in;
+    c.w_out = w_out;
+    return run(c, nullptr, 0, false, stream);
+  }
   const long long T = B * N;
   // Eq. 1: Z = X W_in^T, into y; Eq. 2-3: the mixer, in place; Eq. 4: Y = M W_out^T, in place
   rc = whtmix_project(x, w_in, y, T, C, WHTMIX_BF16, stream);

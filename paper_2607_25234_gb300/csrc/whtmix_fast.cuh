@@ -444,14 +444,15 @@ __device__ __forceinline__ void row_loc(long long b0, long long r, long long lv,
 // Gains as phase 2 reads them, per column: storage position sp of a workspace row, whose element
 // j is logical plane element (j << R) + sigma_inv(sp).  at() is one element of the column, at2()
 // the elements of the storage positions sp and sp + 1 (sp even), which sigma_inv keeps adjacent.
-template <int R>
+// NAT: the workspace rows are in natural order (storage position sp is plane element (j << R) + sp).
+template <int R, bool NAT = false>
 struct FullGain {  // G [N, C] as given
   static constexpr bool SEPARABLE = false;
   const float* g;
   struct Col {
     const float* p;
   };
-  __device__ __forceinline__ Col col(int sp) const { return {g + sigma_inv(sp)}; }
+  __device__ __forceinline__ Col col(int sp) const { return {g + (NAT ? sp : sigma_inv(sp))}; }
   __device__ __forceinline__ float at(const Col& c, long long j) const { return __ldg(c.p + (j << R)); }
   __device__ __forceinline__ float2 at2(const Col& c, long long j) const {
     return __ldg(reinterpret_cast<const float2*>(c.p + (j << R)));

@@ -61,8 +61,11 @@ def test_project_bf16_output_and_in_place(T, C):
     assert torch.equal(x2, z)
 
 
+# (1, 65536, 128), (3, 16384, 128), (2, 32768, 128), (9, 16384, 128), (3, 65536, 128): the fused
+# block kernel (columns of 128, 256, 512 rows; the last two over several plane groups)
 @pytest.mark.parametrize("B,N,C", [(2, 64, 64), (3, 256, 128), (1, 64, 256), (2, 4096, 128), (1, 65536, 128),
-                                   (16, 8192, 256)])
+                                   (16, 8192, 256), (3, 16384, 128), (2, 32768, 128), (9, 16384, 128),
+                                   (3, 65536, 128)])
 def test_block_forward_matches_oracle(B, N, C):
     d = inputs.make_inputs(B, N, C, "bf16", seed=B + N + C)
     w_in = (inputs.normal(90 + C, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32)
