@@ -178,9 +178,11 @@ WHTMIX_API int whtmix_project(const void *x, const void *w, void *z, int64_t T, 
 
 /* The whole mixer block of Section III-B, Eq. 1-4, forward: Z = X W_in^T, M = the mixer of Z with
  * gains G (as whtmix_forward), Y = M W_out^T, per token row; x, y [B, N, C] bf16, w_in, w_out
- * [C, C] bf16 (out, in), gains [N, C] fp32.  Z and M are rounded to bf16 between the steps (the
- * block's activations), arithmetic is fp32.  dtype must be WHTMIX_BF16; C 64, 128 or 256.  y may be
- * x itself.  Three launches on `stream` (projection, mixer, projection), each in place in y. */
+ * [C, C] bf16 (out, in), gains [N, C] fp32; arithmetic is fp32 and M is rounded to bf16 before
+ * W_out (the block's activation).  dtype must be WHTMIX_BF16; C 64, 128 or 256.  y may be x itself.
+ * C = 128 with 2^21 <= N*C <= 2^23: one launch on `stream` (the projections fused into the mixer's
+ * row phases; Z stays fp32).  Other shapes: three launches (projection, mixer, projection), each in
+ * place in y, Z also rounded to bf16. */
 WHTMIX_API int whtmix_block_forward(const void *x, const void *w_in, const void *gains, const void *w_out, void *y,
                                     int64_t B, int64_t N, int64_t C, int dtype, void *stream);
 
