@@ -240,6 +240,26 @@ def reference_arm(args, w):
     print(json.dumps(line), flush=True)
 
 
+def alu_floor(w, sms: int, sm_mhz):
+    """The adds of the transform against the SMs' fp32 lanes: 2 L log2(L) adds (forward, two
+    transforms) and L multiplies per plane; the backward adds 3 L log2(L) + 2 L.  Floor = adds /
+    (SMs x 128 lanes x 2 (packed f32x2 add) x SM clock)."""
+    L = w.N * w.C
+    lg = L.bit_length() - 1
+    adds = 2 * L * lg
+    muls = L
+    if w.backward:
+        adds += 3 * L * lg
+        muls += 2 * L
+    adds *= w.B
+    muls *= w.B
+    if not sm_mhz:
+        return {"adds": adds, "muls": muls, "floor_us": None}
+    floor_s = adds / (sms * 128 * 2 * sm_mhz * 1e6)
+    return {"adds": adds, "muls": muls, "sms": sms, "sm_mhz": sm_mhz, "lanes_per_sm": 128, "packed_f32x2": True,
+            "floor_us": 1e6 * floor_s}
+
+
 def traffic_from_profile(workload: str):
     """dram bytes per launch from a committed ncu summary, only while the kernel sources match."""
     p = os.path.join(ROOT, "profiles", "roofline_traffic.json")
@@ -463,6 +483,10 @@ def ours(args, w):
                          "kernel": kernel_name(w) + (f" + {backward_kernel_name(w)} (two launches per step)" if w.backward
                                                      else " (one launch per step)")},
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K * launches_per_step, "clocks": clocks}
+    alu = alu_floor(w, torch.cuda.get_device_properties(dev).multi_processor_count, clocks.get("sm_mhz"))
+    if alu["floor_us"] is not None:
+        alu["frac_of_step"] = alu["floor_us"] / (elapsed_ms * 1e3 / K)
+    line["alu_floor"] = alu
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
