@@ -56,7 +56,7 @@ def kernel_name(w) -> str:
     if block_fused(w):
         return f"k_block_fast<bf16, R=14, Q={m - 14}>"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
-        r = 14 if m == 23 else 13
+        r = 13
         sep = ", separable gains" if w.gains == "separable" else ""
         pad = ", in-kernel token padding" if w.padded_io else ""
         name = f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}{pad}>"

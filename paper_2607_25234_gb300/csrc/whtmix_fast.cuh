@@ -565,25 +565,49 @@ __device__ __forceinline__ void pair_sync(int quarter) {
   tmem_fence_after();
 }
 
-// Phase 2, TMEM variant (Q = 8, 9).  Per TMEM lane: one column of 2^Q rows; the lane's 2*ET
-// columns hold element k of warp half hw at column hw*ET + k (ET = 2^(Q-1) elements per thread).
-// Bits: k0..k(et-1) local to a thread, k(et) = warp half (traded through TMEM).
+// Column bit 9 for Q = 10, held by lane bit 4: lanes l and l ^ 16 hold the two halves of one
+// column at the same register positions (combinations s = 0..7 of bits 6..8).  A swap trades half
+// of them so that each lane holds both halves for four combinations: afterwards lane bit 4 = h
+// holds combinations 4h + t, t = 0..3, with bit 9 = 0 in v[t] and bit 9 = 1 in v[t + 4].  The
+// same swap restores the layout.  (Half the shuffles of a butterfly across the lanes.)
+template <int W>
+__device__ __forceinline__ void lane16_swap(float2 (&v)[8][W], int h) {
+#pragma unroll
+  for (int t = 0; t < 4; ++t)
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const float2 a = v[t][w], b = v[t + 4][w];
+      const float2 snd = h ? a : b;
+      const float2 r = make_float2(__shfl_xor_sync(0xffffffffu, snd.x, 16), __shfl_xor_sync(0xffffffffu, snd.y, 16));
+      v[t][w] = h ? r : a;
+      v[t + 4][w] = h ? b : r;
+    }
+}
+
+// Phase 2, TMEM variant (Q = 8, 9, 10).  Per TMEM lane: 2^Q rows of one column (Q = 8, 9), or
+// half of a 1024-row column (Q = 10: lanes l and l ^ 16 of a warp share a column, lane bit 4 =
+// column bit 9, so a pass covers 64 columns).  The lane's 2*ET columns hold element k of warp
+// half hw at column hw*ET + k (ET = 2^(Q-1) elements per thread, 2^8 for Q = 10).
+// Bits: k0..k(et-1) local to a thread, k(et) = warp half (traded through TMEM), k9 = lane bit 4.
 //   round A: own ET elements, bits k0..k5 forward (pairs on the top local bit), global -> TMEM
-//   round B: bits k6..k(et) forward, gain, back; each warp half takes k5 = hw
+//   round B: bits k6..k(et) (and k9 after a half swap between the lanes) forward, gain, back;
+//            each warp half takes k5 = hw
 //   round C: own ET elements, bits k0..k5 again, TMEM -> global
 template <int Q, int R, class GainT>
 __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, float scale, int m, long long u_begin,
                                               long long u_end, uint32_t tlane) {
-  constexpr int ET_BITS = Q - 1;                       // 8, 7 for Q = 9, 8
+  constexpr bool LANE_BIT = Q == 10;
+  constexpr int ET_BITS = LANE_BIT ? 8 : Q - 1;        // 8, 7 for Q = 9, 8; 8 for Q = 10
   constexpr int ET = 1 << ET_BITS;
-  constexpr int PER_PASS = 128;                        // columns per pass (one per TMEM lane)
+  constexpr int PER_PASS = LANE_BIT ? 64 : 128;        // columns per pass
   constexpr int ITA = ET / 128;                        // round A/C iterations (64 pairs each)
   constexpr int NH = 1 << (ET_BITS - 5);               // high combinations in round B (incl. warp half)
   constexpr int W = 64 / NH;                           // pairs per high combination
   constexpr int ITB = 16 / W;                          // round B iterations
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int quarter = warp & 3, hw = warp >> 2;
-  const int slot = quarter * 32 + lane;
+  const int slot = LANE_BIT ? quarter * 16 + (lane & 15) : quarter * 32 + lane;
+  const int l4 = LANE_BIT ? (lane >> 4) & 1 : 0;     // column half (rows 512 l4 ...)
   const float2 sc = make_float2(scale, scale);
   for (long long u0 = u_begin; u0 < u_end; u0 += PER_PASS) {
     const long long u = u0 + slot;
@@ -593,7 +617,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
     const int sp = static_cast<int>(uu & ((1 << R) - 1));  // storage position of the column
     float* colp = ws + (b << m) + sp;
     const auto gcol = gain.col(sp);
-    float* own = colp + (static_cast<long long>(hw * ET) << R);
+    float* own = colp + (static_cast<long long>(l4 * 2 * ET + hw * ET) << R);
     // round A
 #pragma unroll 1
     for (int it = 0; it < ITA; ++it) {
@@ -641,10 +665,19 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
           if ((s & hh) == 0)
 #pragma unroll
             for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
+      if constexpr (LANE_BIT) {
+        lane16_swap(v, l4);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+          for (int w = 0; w < W; ++w) bf2(v[t][w], v[t + 4][w]);
+      }
 #pragma unroll
       for (int s = 0; s < NH; ++s) {
         const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-        const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+        // (Q = 10: after the swap, s / 4 is column bit 9 and the warp-half bit is this lane's l4)
+        const long long j0 = LANE_BIT ? s_hw * 2 * ET + l4 * ET + s_local * 64 + 32 * hw + 2 * W * it
+                                      : s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
 #pragma unroll
         for (int w = 0; w < W; ++w) {
           const long long j = j0 + 2 * w;
@@ -654,6 +687,13 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
           else gg = make_float2(__ldg(gcol.p + (j << R)), __ldg(gcol.p + ((j + 1) << R)));
           v[s][w] = mul2(v[s][w], mul2(gg, sc));
         }
+      }
+      if constexpr (LANE_BIT) {
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+          for (int w = 0; w < W; ++w) bf2(v[t][w], v[t + 4][w]);
+        lane16_swap(v, l4);
       }
 #pragma unroll
       for (int hh = 1; hh < NH; hh <<= 1)
@@ -712,7 +752,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 // three phases.  R and Q are template parameters so that every register array has a static size.
 template <int D, int R, int Q, bool SEP>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
-  static_assert((R == 13 && Q >= 1 && Q <= 9) || (R == 14 && Q == 9), "supported row/column split");
+  static_assert((R == 13 && Q >= 1 && Q <= 10) || (R == 14 && Q == 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   GridSync gsync(P.bar, &flag);
