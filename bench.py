@@ -55,6 +55,11 @@ def kernel_name(w) -> str:
     m = (w.N * w.C).bit_length() - 1
     if block_fused(w):
         return f"k_block_fast<bf16, R=14, Q={m - 14}>"
+    padded_ok = w.n_valid is None or (w.n_valid * w.C * (2 if w.dtype == "bf16" else 4)) % 16 == 0
+    if (w.dtype in ("f32", "bf16") and 14 <= m <= 16 and w.gains == "full" and not w.block
+            and (not w.padded_io or padded_ok)):
+        k = max(1, 2 ** (m - 14) // 2)
+        return f"k_forward_cluster<{w.dtype}, column bits {m - 14}> (clusters of {k} CTAs, one plane each)"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 13
         sep = ", separable gains" if w.gains == "separable" else ""

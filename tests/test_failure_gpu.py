@@ -35,7 +35,7 @@ def to_dev(a: np.ndarray, dtype: str) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-@pytest.mark.parametrize("B,N,C,dtype,backward", [(2, 4096, 64, "bf16", False),    # fast forward
+@pytest.mark.parametrize("B,N,C,dtype,backward", [(2, 8192, 128, "bf16", False),   # three-phase fast forward
                                                   (3, 1024, 128, "f32", True),     # fast backward
                                                   (2, 8192, 64, "i32", False)])    # generic engine
 def test_stuck_barrier_times_out_and_the_context_stays_usable(B, N, C, dtype, backward):
