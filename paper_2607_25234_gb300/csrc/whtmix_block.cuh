@@ -356,11 +356,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_block_fast(Params P, const __nv_
     }
     // phase 1: X -> (W_in) -> channel and token transforms -> workspace (row r of the group is
     // plane b0 + (r >> Q), tokens 128 (r mod 2^Q) ...)
-    // The worker's later X tiles are fetched into L2 up front, so that only the first tile's
-    // load waits on HBM; G, first read in phase 2, is fetched into L2 in pieces, one per tile.
-    if (wt == 0)
-      for (long long r = rb + worker + 2; r < re; r += 2)
-        asm volatile("cp.async.bulk.prefetch.L2.global [%0], 32768;" ::"l"(x + (b0 << m) + (r << R)) : "memory");
+    // G, first read in phase 2, is fetched into L2 in pieces, one per tile.  (Fetching the
+    // worker's later X tiles into L2 up front as well: 4 us slower in the phase probe, no change in
+    // the steady-state bench; left out.)
     if (rb + worker < re) stage_x(worker_buf(worker), x + (b0 << m) + ((rb + worker) << R), wt);
     for (long long r = rb + worker; r < re + worker; r += 2) {
       const bool active = r < re && ok;
