@@ -4,8 +4,9 @@
 // Same three phases as the generic plan M (Section III-B map; see whtmix_kernels.cuh), written
 // for the instruction and latency budget of the path: the butterflies need 2 log2(NC) fp32 adds
 // per element, which at N*C = 2^23 on 152 SMs is about as long as streaming X, G and Y through
-// HBM.  A plane of 2^m elements is viewed as 2^Q rows of 2^R contiguous elements (R = 13, or 14
-// for m = 23, so that Q <= 9):
+// HBM.  A plane of 2^m elements is viewed as 2^Q rows of 2^R contiguous elements (R = 13 for the
+// forward launches, Q <= 10; the row code also serves R = 14, used by the backward and the fused
+// block):
 //   phase 1  every row: its R bits forward                              X  -> workspace
 //   phase 2  every column: its Q bits forward, gain G/L, Q bits again   workspace -> workspace
 //   phase 3  every row: its R bits again                                workspace -> Y
@@ -20,7 +21,7 @@
 //   * phase 2 gives columns to threads: whole columns in registers when a column has <= 128
 //     elements; otherwise the two warps (w, w+4) that share a TMEM lane quarter hold one column
 //     per lane (Blackwell tensor memory as per-thread storage, up to 256 fp32 per thread) and
-//     trade the bit between their halves through TMEM;
+//     trade the bit between their halves through TMEM; 1024-row columns take two lanes of a warp;
 //   * column ranges are balanced and aligned to 8 columns (32-byte sectors).
 #pragma once
 
