@@ -415,52 +415,85 @@ def ours(args, w):
     peak, peak_kind = measured_peaks()
     achieved = ideal / (step_ms / 1e3) / 1e9
 
-    # end to end through the public Python API: pinned host buffers, copies inside the timed loop
+    # End to end through the public Python API: every step copies its inputs in from pinned host
+    # memory and its result back out.  Two device buffer sets and three streams (copies in,
+    # compute, copies out) let step i + 1's copies in and step i - 1's copy out run beside step i's
+    # launch, as a serving loop would; events order each buffer set's reuse.
     e2e = None
     if rank == 0 or world > 1:
         xh = x_host.pin_memory()
         gh = g_host.pin_memory()
         yh = torch.empty_like(xh).pin_memory()
-        xd, gd, yd = xs[0], gs[0], ys[0]
-        h2d = [(xd, xh), (gd, gh)]
-        d2h = [(yh, yd)]
-        if w.backward:
-            dyh = dy_host.pin_memory()
-            dxh = torch.empty_like(dyh).pin_memory()
-            dgh = torch.empty_like(gh).pin_memory()
-            h2d.append((dys[0], dyh))
-            d2h += [(dxh, dxs[0]), (dgh, dgs[0])]
-        ke = max(3, min(K, 50))
+        dyh = dy_host.pin_memory() if w.backward else None
+        dxh = torch.empty_like(dyh).pin_memory() if w.backward else None
+        dgh = torch.empty_like(gh).pin_memory() if w.backward else None
+        NB = 2
+        s_in, s_comp, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        ev_in = [torch.cuda.Event() for _ in range(NB)]
+        ev_comp = [torch.cuda.Event() for _ in range(NB)]
+        ev_out = [torch.cuda.Event() for _ in range(NB)]
 
-        def e2e_step():
-            for dst, src in h2d:
-                dst.copy_(src, non_blocking=True)
-            if w.block:
-                whtmix.block_forward(xd, wi, gd, wo, out=yd)
-            elif sep:
-                whtmix.forward_separable(xd, gd[:w.N], gd[w.N:], out=yd)
-            elif w.padded_io:
-                whtmix.forward_padded(xd, gd, out=yd)
-            else:
-                whtmix.forward(xd, gd, out=yd)
+        def copies_in(k):
+            pairs = [(xs[k], xh), (gs[k], gh)]
             if w.backward:
-                whtmix.backward(xd, gd, dys[0], dx=dxs[0], dg=dgs[0])
-            for dst, src in d2h:
-                dst.copy_(src, non_blocking=True)
-        for _ in range(3):
-            e2e_step()
+                pairs.append((dys[k], dyh))
+            return pairs
+
+        def copies_out(k):
+            pairs = [(yh, ys[k])]
+            if w.backward:
+                pairs += [(dxh, dxs[k]), (dgh, dgs[k])]
+            return pairs
+
+        def e2e_step(i):
+            k = i % NB
+            with torch.cuda.stream(s_in):
+                if i >= NB:
+                    s_in.wait_event(ev_comp[k])  # the set's previous inputs are consumed
+                for dst, src in copies_in(k):
+                    dst.copy_(src, non_blocking=True)
+                ev_in[k].record(s_in)
+            with torch.cuda.stream(s_comp):
+                s_comp.wait_event(ev_in[k])
+                if i >= NB:
+                    s_comp.wait_event(ev_out[k])  # the set's previous outputs are copied out
+                xd, gd, yd = xs[k], gs[k], ys[k]
+                if w.block:
+                    whtmix.block_forward(xd, wi, gd, wo, out=yd)
+                elif sep:
+                    whtmix.forward_separable(xd, gd[:w.N], gd[w.N:], out=yd)
+                elif w.padded_io:
+                    whtmix.forward_padded(xd, gd, out=yd)
+                else:
+                    whtmix.forward(xd, gd, out=yd)
+                if w.backward:
+                    whtmix.backward(xd, gd, dys[k], dx=dxs[k], dg=dgs[k])
+                ev_comp[k].record(s_comp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_comp[k])
+                for dst, src in copies_out(k):
+                    dst.copy_(src, non_blocking=True)
+                ev_out[k].record(s_out)
+
+        ke = max(3, min(K, 50))
+        for i in range(4):
+            e2e_step(i)
         torch.cuda.synchronize(dev)
         s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        s2.record(stream)
-        for _ in range(ke):
-            e2e_step()
-        e2.record(stream)
+        s2.record(s_in)
+        for i in range(ke):
+            e2e_step(i)
+        e2.record(s_out)
         torch.cuda.synchronize(dev)
         e2e_ms = s2.elapsed_time(e2) / ke
         e2e = {"value": tokens_per_step / (e2e_ms / 1e3), "unit": "tokens/s",
-               "h2d_bytes_per_step": sum(src.numel() * src.element_size() for _, src in h2d),
-               "d2h_bytes_per_step": sum(dst.numel() * dst.element_size() for dst, _ in d2h),
-               "steps": ke, "ms_per_step": e2e_ms}
+               "h2d_bytes_per_step": sum(src.numel() * src.element_size() for _, src in copies_in(0)),
+               "d2h_bytes_per_step": sum(dst.numel() * dst.element_size() for dst, _ in copies_out(0)),
+               "steps": ke, "ms_per_step": e2e_ms,
+               "pipeline": "copies in, compute, copies out on three streams, two buffer sets"}
+        rc = lib.whtmix_sync(ctypes.c_void_p(int(s_comp.cuda_stream)))
+        if rc != 0:
+            raise whtmix.WhtmixError(rc, "device-side check after the end-to-end loop")
 
     if rank != 0:
         if world > 1:
