@@ -39,9 +39,14 @@ FALLBACK_HBM_GBS = 6800.0
 REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
            0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
            0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
-KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_25234_gb300", "csrc", f) for f in
-                  ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_capi.cu",
-                   "whtmix_block.cuh", "whtmix_block.cu")]
+# The device-code files each kernel family is compiled from: a committed DRAM-traffic figure is
+# used only while the hash of its family's files is unchanged (and only for the kernel it names).
+KERNEL_FAMILY_SOURCES = {
+    "k_forward_fast": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh"),
+    "k_backward_fast": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_fast_bwd.cuh"),
+    "k_block_fast": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_block.cuh", "whtmix_block.cu"),
+    "k_forward_plane": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_plane.cuh", "whtmix_plane.cu"),
+}
 
 
 def block_fused(w) -> bool:
@@ -56,10 +61,9 @@ def kernel_name(w) -> str:
     if block_fused(w):
         return f"k_block_fast<bf16, R=14, Q={m - 14}>"
     padded_ok = w.n_valid is None or (w.n_valid * w.C * (2 if w.dtype == "bf16" else 4)) % 16 == 0
-    if (w.dtype in ("f32", "bf16") and 14 <= m <= 16 and w.gains == "full" and not w.block
-            and (not w.padded_io or padded_ok)):
-        k = max(1, 2 ** (m - 14) // 2)
-        return f"k_forward_cluster<{w.dtype}, column bits {m - 14}> (clusters of {k} CTAs, one plane each)"
+    if (w.dtype in ("f32", "bf16") and 14 <= m <= 16 and (m < 16 or w.B >= 80) and w.gains == "full"
+            and not w.block and (not w.padded_io or padded_ok)):
+        return f"k_forward_plane<{w.dtype}, column bits {m - 14}> (one plane per CTA, in tensor memory)"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 13
         sep = ", separable gains" if w.gains == "separable" else ""
@@ -78,11 +82,16 @@ def backward_kernel_name(w) -> str:
     return "k_backward_s" if m <= 13 else "k_backward_m"
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(kernel: str) -> str:
+    """Hash of the source files of the kernel family `kernel` belongs to ("" if unknown)."""
+    family = next((f for f in KERNEL_FAMILY_SOURCES if kernel.startswith(f)), None)
+    if family is None:
+        return ""
     h = hashlib.sha256()
-    for f in sorted(KERNEL_SOURCES):
-        if os.path.exists(f):
-            h.update(open(f, "rb").read())
+    for f in sorted(KERNEL_FAMILY_SOURCES[family]):
+        path = os.path.join(ROOT, "paper_2607_25234_gb300", "csrc", f)
+        if os.path.exists(path):
+            h.update(open(path, "rb").read())
     return h.hexdigest()[:16]
 
 
@@ -266,14 +275,19 @@ def alu_floor(w, sms: int, sm_mhz):
 
 
 def traffic_from_profile(workload: str):
-    """dram bytes per launch from a committed ncu summary, only while the kernel sources match."""
+    """DRAM bytes per launch from a committed ncu summary, only for the kernel the workload launches and
+    only while that kernel's source files are unchanged."""
     p = os.path.join(ROOT, "profiles", "roofline_traffic.json")
     try:
         d = json.load(open(p))
     except Exception:
         return None
     e = d.get(workload)
-    if not e or e.get("kernel_source_hash") != kernel_source_hash():
+    if not e:
+        return None
+    w = inputs.WORKLOADS.get(workload)
+    launched = kernel_name(w) + (" " + backward_kernel_name(w) if w is not None and w.backward else "") if w else ""
+    if e.get("kernel") not in launched or e.get("kernel_source_hash") != kernel_source_hash(e.get("kernel", "")):
         return None
     return e.get("dram_bytes_per_launch")
 

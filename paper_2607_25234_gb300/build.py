@@ -15,7 +15,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libwhtmix.so")
-SOURCES = ["whtmix_capi.cu", "whtmix_fast_f32.cu", "whtmix_fast_bf16.cu", "whtmix_fast_sep_f32.cu", "whtmix_block.cu", "whtmix_cluster.cu",
+SOURCES = ["whtmix_capi.cu", "whtmix_fast_f32.cu", "whtmix_fast_bf16.cu", "whtmix_fast_sep_f32.cu", "whtmix_block.cu", "whtmix_plane.cu",
            "whtmix_fast_sep_bf16.cu", "whtmix_noalloc.cu", "whtmix_proj.cu"]
 OBJDIR = os.path.join(LIBDIR, "obj")
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"

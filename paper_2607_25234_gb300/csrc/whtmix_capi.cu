@@ -16,12 +16,11 @@
 #include "whtmix_kernels.cuh"
 
 namespace whtmix {
-namespace clu {
-// Cluster forward (whtmix_cluster.cu): fp32 / bf16 planes of 2^14 .. 2^16 elements, full gains.
+namespace pln {
+// One plane per CTA in tensor memory (whtmix_plane.cu): fp32 / bf16 planes of 2^14 .. 2^16 elements.
 cudaError_t forward_f32(const Params& P, cudaStream_t stream);
 cudaError_t forward_bf16(const Params& P, cudaStream_t stream);
-bool usable(int m, bool bf16);  // the cluster shape fits this device (checked once per kernel)
-}  // namespace clu
+}  // namespace pln
 namespace blk {
 // Fused block (whtmix_block.cu): bf16, C = 128, 2^21 <= N C <= 2^23, full gains, N_valid = N.
 cudaError_t forward_bf16(const Params& P, const void* w_in, const void* w_out, int sms, cudaStream_t stream);
@@ -41,6 +40,13 @@ thread_local int g_last_cuda_error = 0;
 
 constexpr size_t HEADER_BYTES = sizeof(GridBarrier);
 constexpr size_t WS_TARGET_BYTES = 64ull << 20;  // plane-group workspace, L2-resident (126 MiB L2)
+constexpr int64_t PLANE_MIN_BATCH_16 = 80;
+// Smallest batch for which the one-plane-per-CTA forward beats the three-phase kernel: a plane of
+// 2^16 elements is four rows for one CTA (two per worker, one after the other), so a small batch
+// leaves most SMs idle (measured on [B, 512, 128] bf16, back to back: B = 64 three-phase 24.6 us
+// against 26.6, B = 96 30.8 against 26.7, B = 128 36.0 against 28.7); 2^14 and 2^15 planes are one
+// row per worker.
+int64_t plane_kernel_min_batch(int m) { return m == 16 ? PLANE_MIN_BATCH_16 : 1; }
 
 int cuda_fail(cudaError_t e) {
   g_last_cuda_error = static_cast<int>(e);
@@ -483,27 +489,24 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
   if (use_user_ws) {
     if (!user_ws || (reinterpret_cast<uintptr_t>(user_ws) & 255u) || user_ws_bytes < lay.total) return WHTMIX_ERR_WORKSPACE;
   }
-  // Planes of 2^14 .. 2^16 elements: one cluster (1 or 2 CTAs) per plane, the fp32 intermediate in
-  // the cluster's shared memory, no workspace.  (The cluster kernel covers up to 2^19 with clusters
-  // of up to 16 CTAs, but from 2^17 on the three-phase kernel is faster: measured at
-  // [32, 4096, 64] f32, 74.7 against 49.5 us.)
+  // Planes of 2^14 .. 2^16 elements: one plane per CTA, the fp32 intermediate in the SM's tensor
+  // memory, no workspace and no device-wide barrier.
   if (!c.backward && !c.separable && !c.w_in && c.dtype != WHTMIX_I32 && m >= 14 && m <= 16 &&
-      (lv == L || (lv * es) % 16 == 0)) {
+      c.B >= plane_kernel_min_batch(m) && (lv == L || (lv * es) % 16 == 0) &&
+      c.B <= 0x7fffffff) {  // one CTA per plane: B fits a grid
     int dev = 0, sms = 0;
     rc = device_check(&dev, &sms);
     if (rc != WHTMIX_OK) return rc;
-    if (clu::usable(m, c.dtype == WHTMIX_BF16)) {
-      Params P{};
-      P.x = c.x;
-      P.g = c.g;
-      P.y = c.out;
-      P.B = c.B;
-      P.m = m;
-      P.scale = 1.0f / static_cast<float>(L);
-      P.lv = static_cast<long long>(lv);
-      const cudaError_t e = c.dtype == WHTMIX_BF16 ? clu::forward_bf16(P, stream) : clu::forward_f32(P, stream);
-      return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
-    }
+    Params P{};
+    P.x = c.x;
+    P.g = c.g;
+    P.y = c.out;
+    P.B = c.B;
+    P.m = m;
+    P.scale = 1.0f / static_cast<float>(L);
+    P.lv = static_cast<long long>(lv);
+    const cudaError_t e = c.dtype == WHTMIX_BF16 ? pln::forward_bf16(P, stream) : pln::forward_f32(P, stream);
+    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
   }
   int dev = 0, sms = 0;
   rc = device_check(&dev, &sms);
