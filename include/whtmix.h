@@ -203,8 +203,8 @@ WHTMIX_API int whtmix_last_cuda_error(void);
 
 /* Which kernel plan a shape uses: 1 = one tile per plane group (N*C <= 2^13), 2 = three
  * passes through the workspace (2^13 < N*C <= 2^26); 0 for an invalid shape.  (The fp32 / bf16
- * forward of a 2^14..2^16-element plane with full gains runs one plane per thread-block cluster
- * instead, in the cluster's shared memory, without the workspace.) */
+ * forward of a 2^14- or 2^15-element plane with full gains, and of a 2^16-element plane in batches of
+ * 80 or more, runs one plane per CTA instead, in the SM's tensor memory, without the workspace.) */
 WHTMIX_API int whtmix_plan(int64_t N, int64_t C);
 
 #ifdef __cplusplus
