@@ -125,10 +125,10 @@ def test_train_16x8192x256_bf16_forward_backward():
 SWEEP = [(1, 1, 1), (3, 1, 1), (5, 1, 8), (7, 8, 1), (3, 2, 2), (9, 4, 16), (2, 16, 4), (33, 32, 8),
          (3, 64, 128), (2, 128, 64), (1, 8192, 1), (1, 1, 8192), (2, 1, 16384), (3, 16384, 1),
          (2, 64, 256), (3, 512, 32), (1, 2048, 64), (2, 256, 1024), (1, 1 << 18, 2), (1, 2, 1 << 18),
-         # every plane size of the cluster forward (2^14, 2^15, 2^16: clusters of 1, 1, 2 CTAs) and
-         # every column height of the three-phase forward (2^17 .. 2^23, Q = 4 .. 10)
-         # (2^17, 2^18, 2^19 above)
-         (3, 2048, 8), (2, 128, 256), (3, 512, 128), (1, 65536, 1),
+         # every plane size of the one-plane-per-CTA forward (2^14, 2^15; 2^16 from a batch of 80:
+         # smaller batches of 2^16 planes run three-phase) and every column height of the
+         # three-phase forward (2^16 .. 2^23, Q = 3 .. 10; 2^17, 2^18, 2^19 above)
+         (3, 2048, 8), (2, 128, 256), (80, 256, 256), (3, 512, 128), (1, 65536, 1),
          (2, 1024, 1024), (3, 256, 4096), (1, 4096, 512), (1, 4096, 1024), (2, 8192, 512),
          (1, 1 << 20, 8), (1, 16, 1 << 19)]
 
@@ -173,8 +173,8 @@ def test_integer_mode_wraps_mod_2_32():
 
 
 def test_in_place_forward_and_backward():
-    # single tile, cluster forward (clusters of 2), three-phase forward
-    for (B, N, C) in [(3, 64, 64), (2, 512, 128), (2, 1024, 128)]:
+    # single tile, one plane per CTA (2^15), three-phase forward
+    for (B, N, C) in [(3, 64, 64), (2, 256, 128), (2, 1024, 128)]:
         d = inputs.make_inputs(B, N, C, "f32", seed=6, with_dy=True)
         x = to_dev(d["x"], "f32")
         g = to_dev(d["g"], "f32")
