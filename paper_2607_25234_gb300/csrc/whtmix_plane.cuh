@@ -5,8 +5,9 @@
 // A plane is NR = 2^CB rows of 2^14 elements (CB = m - 14 <= 2); a CTA has two row workers of 128
 // threads and TMEM's 512 columns x 128 lanes (256 KiB) hold up to four fp32 rows: row r lives in
 // columns [256 (r mod 2) + 128 (r / 2), +128) of the lanes of worker r mod 2, thread wt in lane wt.
-//   phase 1  each worker, for each of its rows: X row -> 14 row bits in registers and one exchange
-//            through its shared-memory buffer -> the thread's 64 pairs into its TMEM lane;
+//   phase 1  each worker, for each of its rows (the next one prefetched by cp.async): X row -> 14
+//            row bits in registers and one exchange through its shared-memory buffer -> the
+//            thread's 64 pairs into its TMEM lane;
 //   phase 2  thread wt of either worker meets the same 128 row positions of every row of the
 //            plane in its lane (both workers' warps w and w + 4 reach the lane): the CB column
 //            bits, the gain G/L and the CB bits back, half the pairs each;
@@ -38,7 +39,9 @@ using fast::THREADS;          // 256: workers 0 (warps 0-3) and 1 (warps 4-7)
 constexpr int R = 14;         // row bits
 constexpr int WK = 128;       // threads per row worker
 constexpr int ROW = 1 << R;   // elements per row
-constexpr size_t SMEM_BYTES = 2 * ROW * sizeof(float);  // one exchange buffer per worker (> half an SM)
+constexpr int STG = 64 * WK;   // staging floats per worker: a bf16 row, or the first half of an fp32 row
+// an exchange buffer and a staging area per worker (more than half an SM: one CTA per SM)
+constexpr size_t SMEM_BYTES = 2 * (ROW + STG) * sizeof(float);
 
 // TMEM column of pair s's x (y at + 64) for row r of the plane, in this thread's lane.
 __device__ __forceinline__ uint32_t row_col(int r) { return 256u * (r & 1) + 128u * (r >> 1); }
@@ -70,19 +73,45 @@ __device__ __forceinline__ void pairs_from_tmem(uint32_t ta, float2 (&b)[64]) {
   fast::tmem_wait_ld();
 }
 
-// Phase 1 row: X (elements e0 ..., lim of them stored) -> the 14 row bits -> this thread's pairs
-// into TMEM at ta (rounds as the three-phase forward's rows).
+// Phase 1 row: X (elements e0 ..., lim of them stored; a whole bf16 row or the first half of an
+// fp32 row already staged in stg by cp.async) -> the 14 row bits -> this thread's pairs into TMEM
+// at ta (rounds as the three-phase forward's rows).  Once the row is in registers the worker's
+// next row (src_next, if not null) is staged behind it.  Each thread reads back only the chunks it
+// copied, so the staging area needs no barrier.
 template <int D>
-__device__ __forceinline__ void row_in(const void* src, long long e0, int lim, float* buf, int wt, int worker,
-                                       uint32_t ta) {
+__device__ __forceinline__ void row_in(const void* src, long long e0, int lim, float* buf, float* stg, int wt,
+                                       int worker, uint32_t ta, const void* src_next, long long e0_next, int lim_next) {
   constexpr int VS = ROW / 16;
   float2 a[16][4];
+  if constexpr (D == DT_F32) {
 #pragma unroll
-  for (int v = 0; v < 16; ++v) {
-    const int o = 8 * wt + VS * v;
-    ld8_pad<D>(src, e0 + (o < lim ? o : 0), a[v], lim - o);
+    for (int v = 8; v < 16; ++v) {
+      const int o = 8 * wt + VS * v;
+      ld8_pad<D>(src, e0 + (o < lim ? o : 0), a[v], lim - o);
+    }
+  }
+  fast::cp_async_wait_all();
+  if constexpr (D == DT_BF16) {
+#pragma unroll
+    for (int v = 0; v < 16; ++v) {
+      const uint4 u = *reinterpret_cast<const uint4*>(stg + (v * WK + wt) * 4);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[v][i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+    }
+  } else {
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const float4 q0 = *reinterpret_cast<const float4*>(stg + ((2 * v) * WK + wt) * 4);
+      const float4 q1 = *reinterpret_cast<const float4*>(stg + ((2 * v + 1) * WK + wt) * 4);
+      a[v][0] = make_float2(q0.x, q0.y);
+      a[v][1] = make_float2(q0.z, q0.w);
+      a[v][2] = make_float2(q1.x, q1.y);
+      a[v][3] = make_float2(q1.z, q1.w);
+    }
   }
   fast::round_v(a);
+  if (src_next != nullptr) fast::stage_row_in<D, R>(src_next, e0_next, stg, wt, lim_next);
 #pragma unroll
   for (int v = 0; v < 16; ++v)
 #pragma unroll
@@ -210,17 +239,25 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_plane(Params P) {
   const long long b = blockIdx.x;
   const int worker = threadIdx.x / WK, wt = threadIdx.x % WK;
   float* buf = pl_smem + worker * ROW;
+  float* stg = pl_smem + 2 * ROW + worker * STG;
   if (threadIdx.x < 32) fast::tmem_alloc_512(&tmem_slot);
   fast::tmem_fence_before();
   __syncthreads();
   fast::tmem_fence_after();
   // this thread's lane: warps w and w + 4 (thread wt of either worker) share lane wt
   const uint32_t lane_ta = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16);
-  for (int r = worker; r < NR; r += 2) {
+  if (worker < NR) {
     long long e0;
     int lim;
+    fast::row_loc<R, CB>(0, b * NR + worker, P.lv, &e0, &lim);
+    fast::stage_row_in<D, R>(P.x, e0, stg, wt, lim);
+  }
+  for (int r = worker; r < NR; r += 2) {
+    long long e0, e0n = 0;
+    int lim, limn = 0;
     fast::row_loc<R, CB>(0, b * NR + r, P.lv, &e0, &lim);
-    row_in<D>(P.x, e0, lim, buf, wt, worker, lane_ta + row_col(r));
+    if (r + 2 < NR) fast::row_loc<R, CB>(0, b * NR + r + 2, P.lv, &e0n, &limn);
+    row_in<D>(P.x, e0, lim, buf, stg, wt, worker, lane_ta + row_col(r), r + 2 < NR ? P.x : nullptr, e0n, limn);
   }
   tmem_cta_sync();  // every row of the plane is in TMEM
   columns<CB>(lane_ta, static_cast<const float*>(P.g), P.scale, wt, worker);
