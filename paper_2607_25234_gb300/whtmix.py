@@ -17,7 +17,8 @@ import torch
 
 from . import build as _build
 
-__all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_separable", "backward_separable",
+__all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_noalloc", "forward_separable",
+           "backward_separable",
            "forward_padded", "backward_padded", "project", "block_forward",
            "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
            "WHTMixSeparableFunction", "pad_tokens", "EXPORTS", "library"]
@@ -60,6 +61,7 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_forward.argtypes = [p, p, p, i64, i64, i64, i, p]
             lib.whtmix_backward.argtypes = [p, p, p, p, p, i64, i64, i64, i, p]
             lib.whtmix_forward_ex.argtypes = [p, p, p, i64, i64, i64, i, p, sz, p]
+            lib.whtmix_forward_noalloc.argtypes = [p, p, p, i64, i64, i64, i, p]
             lib.whtmix_backward_ex.argtypes = [p, p, p, p, p, i64, i64, i64, i, p, sz, p]
             lib.whtmix_workspace_bytes.argtypes = [i64, i64, i64, i, i, ctypes.POINTER(sz)]
             lib.whtmix_sync.argtypes = [p]
@@ -88,9 +90,32 @@ def _check(rc: int, what: str):
         raise WhtmixError(rc, what)
 
 
-def _stream_ptr(stream) -> int:
-    s = stream if stream is not None else torch.cuda.current_stream()
-    return int(s.cuda_stream)
+def _call(what: str, device: torch.device, stream, fn, *args) -> None:
+    """Runs one entry point with ``device`` current, on ``stream`` (default: the device's current
+    stream, appended as the last argument); raises WhtmixError on a nonzero status."""
+    with torch.cuda.device(device):
+        s = stream if stream is not None else torch.cuda.current_stream(device)
+        if s.device != device:
+            raise ValueError(f"stream is on {s.device}, the tensors on {device}")
+        _check(fn(*args, int(s.cuda_stream)), what)
+
+
+def _on_device(t: torch.Tensor, device: torch.device, name: str) -> None:
+    if not t.is_cuda or t.device != device:
+        raise ValueError(f"{name} must be a CUDA tensor on {device} (WHTMix runs on CUDA tensors only)")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _out(t: torch.Tensor | None, shape, dtype: torch.dtype, device: torch.device, name: str) -> torch.Tensor:
+    """A result tensor: a new one, or the caller's, checked to be exactly what the library writes
+    (the C ABI receives only its pointer)."""
+    if t is None:
+        return torch.empty(tuple(shape), dtype=dtype, device=device)
+    if t.dtype != dtype or tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must be {dtype} {list(shape)}, got {t.dtype} {list(t.shape)}")
+    _on_device(t, device, name)
+    return t
 
 
 def _shape(x: torch.Tensor):
@@ -110,21 +135,27 @@ def _check_tensors(x: torch.Tensor, g: torch.Tensor, *others: torch.Tensor):
     if tuple(g.shape) != (N, C):
         raise ValueError(f"gains must be [N, C] = [{N}, {C}], got {tuple(g.shape)}")
     for t in (x, g) + others:
-        if not t.is_cuda:
-            raise ValueError("WHTMix runs on CUDA tensors only")
-        if not t.is_contiguous():
-            raise ValueError("tensors must be contiguous")
+        _on_device(t, x.device, "every tensor")
     return B, N, C
 
 
 def forward(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """Y = H_N (G (.) H_N X H_C) H_C / (N C) per plane (unnormalised, mod 2^32, for int32)."""
     B, N, C = _check_tensors(x, g)
-    y = torch.empty_like(x) if out is None else out
-    if y.shape != x.shape or y.dtype != x.dtype:
-        raise ValueError("out must match x in shape and dtype")
-    _check(library().whtmix_forward(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype],
-                                    _stream_ptr(stream)), "whtmix_forward")
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward", x.device, stream, library().whtmix_forward, x.data_ptr(), g.data_ptr(), y.data_ptr(),
+          B, N, C, DTYPE_CODE[x.dtype])
+    return y
+
+
+def forward_noalloc(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """forward without any device allocation: planes of more than 2^22 elements raise WORKSPACE.
+    Calls share one fixed scratch array per device, so order them on one stream; make the first
+    call on a device outside any stream capture."""
+    B, N, C = _check_tensors(x, g)
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward_noalloc", x.device, stream, library().whtmix_forward_noalloc, x.data_ptr(), g.data_ptr(),
+          y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype])
     return y
 
 
@@ -134,10 +165,10 @@ def backward(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torch.Tenso
     B, N, C = _check_tensors(x, g, dy)
     if dy.shape != x.shape or dy.dtype != x.dtype:
         raise ValueError("dy must match x in shape and dtype")
-    dx = torch.empty_like(dy) if dx is None else dx
-    dg = torch.empty_like(g) if dg is None else dg
-    _check(library().whtmix_backward(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
-                                     B, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_backward")
+    dx = _out(dx, x.shape, x.dtype, x.device, "dx")
+    dg = _out(dg, g.shape, g.dtype, x.device, "dg")
+    _call("whtmix_backward", x.device, stream, library().whtmix_backward, x.data_ptr(), g.data_ptr(), dy.data_ptr(),
+          dx.data_ptr(), dg.data_ptr(), B, N, C, DTYPE_CODE[x.dtype])
     return dx, dg
 
 
@@ -154,10 +185,7 @@ def _check_log_gains(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, *oth
     if tuple(g_c.shape) != (C,):
         raise ValueError(f"log gains must be g_t [{N}] and g_c [{C}], got {tuple(g_t.shape)} and {tuple(g_c.shape)}")
     for t in (x, g_t, g_c) + others:
-        if not t.is_cuda:
-            raise ValueError("WHTMix runs on CUDA tensors only")
-        if not t.is_contiguous():
-            raise ValueError("tensors must be contiguous")
+        _on_device(t, x.device, "every tensor")
     return B, n_valid, N, C
 
 
@@ -167,12 +195,9 @@ def forward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, out
     G[n, c] = exp(g_t[n]) exp(g_c[c]).  When x has fewer tokens than g_t (not a power of two), the
     planes are zero-padded to len(g_t) tokens inside the library and y keeps x's tokens."""
     B, n_valid, N, C = _check_log_gains(x, g_t, g_c)
-    y = torch.empty_like(x) if out is None else out
-    if y.shape != x.shape or y.dtype != x.dtype:
-        raise ValueError("out must match x in shape and dtype")
-    _check(library().whtmix_forward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), y.data_ptr(), B, n_valid,
-                                              N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
-           "whtmix_forward_separable")
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward_separable", x.device, stream, library().whtmix_forward_separable, x.data_ptr(),
+          g_t.data_ptr(), g_c.data_ptr(), y.data_ptr(), B, n_valid, N, C, DTYPE_CODE[x.dtype])
     return y
 
 
@@ -183,13 +208,12 @@ def backward_separable(x: torch.Tensor, g_t: torch.Tensor, g_c: torch.Tensor, dy
     B, n_valid, N, C = _check_log_gains(x, g_t, g_c, dy)
     if dy.shape != x.shape or dy.dtype != x.dtype:
         raise ValueError("dy must match x in shape and dtype")
-    dx = torch.empty_like(dy) if dx is None else dx
-    dg_t = torch.empty_like(g_t) if dg_t is None else dg_t
-    dg_c = torch.empty_like(g_c) if dg_c is None else dg_c
-    _check(library().whtmix_backward_separable(x.data_ptr(), g_t.data_ptr(), g_c.data_ptr(), dy.data_ptr(),
-                                               dx.data_ptr(), dg_t.data_ptr(), dg_c.data_ptr(), B, n_valid, N, C,
-                                               DTYPE_CODE[x.dtype], _stream_ptr(stream)),
-           "whtmix_backward_separable")
+    dx = _out(dx, x.shape, x.dtype, x.device, "dx")
+    dg_t = _out(dg_t, g_t.shape, g_t.dtype, x.device, "dg_t")
+    dg_c = _out(dg_c, g_c.shape, g_c.dtype, x.device, "dg_c")
+    _call("whtmix_backward_separable", x.device, stream, library().whtmix_backward_separable, x.data_ptr(),
+          g_t.data_ptr(), g_c.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg_t.data_ptr(), dg_c.data_ptr(), B,
+          n_valid, N, C, DTYPE_CODE[x.dtype])
     return dx, dg_t, dg_c
 
 
@@ -204,10 +228,7 @@ def _check_padded(x: torch.Tensor, g: torch.Tensor, *others: torch.Tensor):
     if N & (N - 1) or N < max(n_valid, 1):
         raise ValueError(f"gains must have a power-of-two token count >= the {n_valid} tokens of x, got {N}")
     for t in (x, g) + others:
-        if not t.is_cuda:
-            raise ValueError("WHTMix runs on CUDA tensors only")
-        if not t.is_contiguous():
-            raise ValueError("tensors must be contiguous")
+        _on_device(t, x.device, "every tensor")
     return B, n_valid, N, C
 
 
@@ -215,11 +236,9 @@ def forward_padded(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = 
     """The forward on planes zero-padded from x's N_valid tokens to g's N (a power of two), inside the
     library; y keeps x's N_valid tokens (Section III-B: pad before H_N, discard the padded outputs)."""
     B, n_valid, N, C = _check_padded(x, g)
-    y = torch.empty_like(x) if out is None else out
-    if y.shape != x.shape or y.dtype != x.dtype:
-        raise ValueError("out must match x in shape and dtype")
-    _check(library().whtmix_forward_padded(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, n_valid, N, C,
-                                           DTYPE_CODE[x.dtype], _stream_ptr(stream)), "whtmix_forward_padded")
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward_padded", x.device, stream, library().whtmix_forward_padded, x.data_ptr(), g.data_ptr(),
+          y.data_ptr(), B, n_valid, N, C, DTYPE_CODE[x.dtype])
     return y
 
 
@@ -229,11 +248,10 @@ def backward_padded(x: torch.Tensor, g: torch.Tensor, dy: torch.Tensor, dx: torc
     B, n_valid, N, C = _check_padded(x, g, dy)
     if dy.shape != x.shape or dy.dtype != x.dtype:
         raise ValueError("dy must match x in shape and dtype")
-    dx = torch.empty_like(dy) if dx is None else dx
-    dg = torch.empty_like(g) if dg is None else dg
-    _check(library().whtmix_backward_padded(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
-                                            B, n_valid, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
-           "whtmix_backward_padded")
+    dx = _out(dx, x.shape, x.dtype, x.device, "dx")
+    dg = _out(dg, g.shape, g.dtype, x.device, "dg")
+    _call("whtmix_backward_padded", x.device, stream, library().whtmix_backward_padded, x.data_ptr(), g.data_ptr(),
+          dy.data_ptr(), dx.data_ptr(), dg.data_ptr(), B, n_valid, N, C, DTYPE_CODE[x.dtype])
     return dx, dg
 
 
@@ -242,15 +260,16 @@ def project(x: torch.Tensor, w: torch.Tensor, out_dtype: torch.dtype = torch.bfl
     """z = x w^T per token on the tensor cores (x [..., C] bf16, w [C, C] bf16 as (out, in))."""
     if x.dtype != torch.bfloat16 or w.dtype != torch.bfloat16:
         raise TypeError("project takes bfloat16 x and w")
+    if out_dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError(f"project writes float32 or bfloat16, not {out_dtype}")
     C = x.shape[-1]
     if tuple(w.shape) != (C, C):
         raise ValueError(f"w must be [{C}, {C}]")
     for t in (x, w):
-        if not t.is_cuda or not t.is_contiguous():
-            raise ValueError("x and w must be contiguous CUDA tensors")
-    z = torch.empty(x.shape, dtype=out_dtype, device=x.device) if out is None else out
-    _check(library().whtmix_project(x.data_ptr(), w.data_ptr(), z.data_ptr(), x.numel() // C, C,
-                                    DTYPE_CODE[out_dtype], _stream_ptr(stream)), "whtmix_project")
+        _on_device(t, x.device, "x and w")
+    z = _out(out, x.shape, out_dtype, x.device, "out")
+    _call("whtmix_project", x.device, stream, library().whtmix_project, x.data_ptr(), w.data_ptr(), z.data_ptr(),
+          x.numel() // C, C, DTYPE_CODE[out_dtype])
     return z
 
 
@@ -259,12 +278,12 @@ def block_forward(x: torch.Tensor, w_in: torch.Tensor, g: torch.Tensor, w_out: t
     """The mixer block of Section III-B, Eq. 1-4: Y = mix(X W_in^T) W_out^T (bf16)."""
     B, N, C = _check_tensors(x, g)
     for t in (w_in, w_out):
-        if t.dtype != torch.bfloat16 or tuple(t.shape) != (C, C) or not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"w_in and w_out must be contiguous bfloat16 CUDA tensors [{C}, {C}]")
-    y = torch.empty_like(x) if out is None else out
-    _check(library().whtmix_block_forward(x.data_ptr(), w_in.data_ptr(), g.data_ptr(), w_out.data_ptr(),
-                                          y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype], _stream_ptr(stream)),
-           "whtmix_block_forward")
+        if t.dtype != torch.bfloat16 or tuple(t.shape) != (C, C):
+            raise ValueError(f"w_in and w_out must be bfloat16 [{C}, {C}]")
+        _on_device(t, x.device, "w_in and w_out")
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_block_forward", x.device, stream, library().whtmix_block_forward, x.data_ptr(), w_in.data_ptr(),
+          g.data_ptr(), w_out.data_ptr(), y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype])
     return y
 
 
@@ -276,28 +295,32 @@ def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool =
 
 
 def forward_ex(x, g, workspace: torch.Tensor, out=None, stream=None):
+    """forward with a caller-owned workspace of at least workspace_bytes(...) bytes."""
     B, N, C = _check_tensors(x, g, workspace)
-    y = torch.empty_like(x) if out is None else out
-    _check(library().whtmix_forward_ex(x.data_ptr(), g.data_ptr(), y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype],
-                                       workspace.data_ptr(), workspace.numel() * workspace.element_size(),
-                                       _stream_ptr(stream)), "whtmix_forward_ex")
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward_ex", x.device, stream, library().whtmix_forward_ex, x.data_ptr(), g.data_ptr(),
+          y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype], workspace.data_ptr(),
+          workspace.numel() * workspace.element_size())
     return y
 
 
 def backward_ex(x, g, dy, workspace: torch.Tensor, dx=None, dg=None, stream=None):
+    """backward with a caller-owned workspace of at least workspace_bytes(..., backward=True) bytes."""
     B, N, C = _check_tensors(x, g, dy, workspace)
-    dx = torch.empty_like(dy) if dx is None else dx
-    dg = torch.empty_like(g) if dg is None else dg
-    _check(library().whtmix_backward_ex(x.data_ptr(), g.data_ptr(), dy.data_ptr(), dx.data_ptr(), dg.data_ptr(),
-                                        B, N, C, DTYPE_CODE[x.dtype], workspace.data_ptr(),
-                                        workspace.numel() * workspace.element_size(), _stream_ptr(stream)),
-           "whtmix_backward_ex")
+    if dy.shape != x.shape or dy.dtype != x.dtype:
+        raise ValueError("dy must match x in shape and dtype")
+    dx = _out(dx, x.shape, x.dtype, x.device, "dx")
+    dg = _out(dg, g.shape, g.dtype, x.device, "dg")
+    _call("whtmix_backward_ex", x.device, stream, library().whtmix_backward_ex, x.data_ptr(), g.data_ptr(),
+          dy.data_ptr(), dx.data_ptr(), dg.data_ptr(), B, N, C, DTYPE_CODE[x.dtype], workspace.data_ptr(),
+          workspace.numel() * workspace.element_size())
     return dx, dg
 
 
 def sync(stream=None) -> None:
     """Synchronise the stream and raise if a device-side bounded wait expired."""
-    _check(library().whtmix_sync(_stream_ptr(stream)), "whtmix_sync")
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _call("whtmix_sync", s.device, s, library().whtmix_sync)
 
 
 def release_workspaces() -> None:
@@ -324,8 +347,9 @@ class WHTMixFunction(torch.autograd.Function):
 
     @staticmethod
     def forward(ctx, x, g):
+        x, g = x.contiguous(), g.contiguous()
         ctx.save_for_backward(x, g)
-        return forward(x.contiguous(), g.contiguous())
+        return forward(x, g)
 
     @staticmethod
     def backward(ctx, dy):
@@ -339,8 +363,9 @@ class WHTMixSeparableFunction(torch.autograd.Function):
 
     @staticmethod
     def forward(ctx, x, g_t, g_c):
+        x, g_t, g_c = x.contiguous(), g_t.contiguous(), g_c.contiguous()
         ctx.save_for_backward(x, g_t, g_c)
-        return forward_separable(x.contiguous(), g_t.contiguous(), g_c.contiguous())
+        return forward_separable(x, g_t, g_c)
 
     @staticmethod
     def backward(ctx, dy):

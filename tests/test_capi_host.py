@@ -201,3 +201,45 @@ def test_project_and_block_reject_invalid_arguments_before_any_device_work(lib):
     assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 5 * FAKE, 1, 4, 32, 1, None) == 2   # C 64, 128 or 256
     assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 2 * FAKE, 1, 4, 64, 1, None) == 5   # y over w_in
     assert Bk(FAKE, 2 * FAKE, 3 * FAKE, 4 * FAKE, 5 * FAKE, 0, 4, 64, 1, None) == 0
+
+
+def test_binding_refuses_cpu_tensors_and_malformed_outputs(monkeypatch):
+    """The torch binding has no CPU path: every public op raises on CPU tensors before it reaches
+    the library, and a caller-supplied output must be exactly the tensor the library writes."""
+    import torch
+
+    def no_library(*_a, **_k):
+        raise AssertionError("the library was reached")
+
+    monkeypatch.setattr(whtmix, "library", no_library)
+    x = torch.zeros(2, 16, 8)
+    g = torch.ones(16, 8)
+    xb = x.to(torch.bfloat16)
+    w = torch.zeros(8, 8, dtype=torch.bfloat16)
+    gt, gc = torch.zeros(16), torch.zeros(8)
+    calls = [
+        lambda: whtmix.forward(x, g),
+        lambda: whtmix.forward_noalloc(x, g),
+        lambda: whtmix.backward(x, g, x),
+        lambda: whtmix.forward_ex(x, g, torch.zeros(64)),
+        lambda: whtmix.backward_ex(x, g, x, torch.zeros(64)),
+        lambda: whtmix.forward_padded(x[:, :12], g),
+        lambda: whtmix.backward_padded(x[:, :12].contiguous(), g, x[:, :12].contiguous()),
+        lambda: whtmix.forward_separable(x, gt, gc),
+        lambda: whtmix.backward_separable(x, gt, gc, x),
+        lambda: whtmix.project(xb, w),
+        lambda: whtmix.block_forward(xb, w, g, w),
+        lambda: whtmix.WHTMixFunction.apply(x, g),
+    ]
+    for call in calls:
+        with pytest.raises(ValueError, match="CUDA"):
+            call()
+
+    dev = torch.device("cpu")
+    assert whtmix._out(None, (2, 3), torch.float32, dev, "out").shape == (2, 3)
+    with pytest.raises(ValueError, match=r"out must be torch.float32 \[2, 3\]"):
+        whtmix._out(torch.zeros(3, 2), (2, 3), torch.float32, dev, "out")
+    with pytest.raises(ValueError, match="dx must be torch.bfloat16"):
+        whtmix._out(torch.zeros(2, 3), (2, 3), torch.bfloat16, dev, "dx")
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        whtmix._out(torch.zeros(2, 3), (2, 3), torch.float32, dev, "out")

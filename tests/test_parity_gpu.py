@@ -244,6 +244,41 @@ def test_empty_batch_and_errors_on_gpu():
         whtmix.forward(torch.zeros(1, 16, 16), torch.zeros(16, 16))
 
 
+def test_binding_rejects_malformed_outputs_before_any_launch():
+    """The C ABI receives only an output's pointer, so the binding checks the tensor: a result
+    buffer of the wrong shape, dtype, device or layout raises and leaves every buffer untouched."""
+    x = torch.randn(2, 64, 32, device="cuda")
+    g = torch.ones(64, 32, device="cuda")
+    sentinel = torch.full((2, 64, 32), 5.0, device="cuda")
+    bad_outs = [torch.empty(2, 64, 16, device="cuda"), torch.empty(2, 64, 32, device="cuda", dtype=torch.bfloat16),
+                torch.empty(2, 64, 32), torch.empty(2, 32, 64, device="cuda").transpose(1, 2)]
+    for bad in bad_outs:
+        with pytest.raises(ValueError):
+            whtmix.forward(x, g, out=bad)
+        with pytest.raises(ValueError):
+            whtmix.backward(x, g, x, dx=bad)
+    with pytest.raises(ValueError):
+        whtmix.backward(x, g, x, dx=sentinel, dg=torch.empty(64, 16, device="cuda"))
+    with pytest.raises(ValueError):
+        whtmix.forward(x, g, stream=torch.cuda.Stream(device="cuda"), out=torch.empty(2, 64, 8, device="cuda"))
+    torch.cuda.synchronize()
+    assert torch.all(sentinel == 5.0)
+
+
+@pytest.mark.parametrize("B,N,C,dtype", [(2, 64, 32, "f32"), (1, 1024, 128, "bf16"), (3, 4096, 64, "f32"),
+                                         (2, 512, 64, "i32")])
+def test_forward_noalloc_binding(B, N, C, dtype):
+    d = inputs.make_inputs(B, N, C, dtype, seed=21)
+    x, g = to_dev(d["x"], dtype), to_dev(d["g"], "f32" if dtype != "i32" else "i32")
+    y = whtmix.forward_noalloc(x, g)
+    whtmix.sync()
+    r = ref_inputs(d, dtype)
+    assert_close(y, oracle.forward(r["x"], r["g"]), dtype, f"noalloc Y [{B},{N},{C}] {dtype}")
+    with pytest.raises(whtmix.WhtmixError) as e:   # 2^23 elements: beyond the fixed scratch
+        whtmix.forward_noalloc(torch.zeros(1, 65536, 128, device="cuda"), torch.ones(65536, 128, device="cuda"))
+    assert e.value.status == 9
+
+
 def test_autograd_function():
     B, N, C = 2, 256, 64
     d = inputs.make_inputs(B, N, C, "f32", seed=11, with_dy=True)
