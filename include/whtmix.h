@@ -30,7 +30,7 @@
  *                            operation wraps modulo 2^32 -- the result is exact and independent
  *                            of the order of the butterfly stages.
  *   Shapes      B >= 0, N >= 1 and C >= 1 powers of two, N*C <= 2^26 elements per plane,
- *               B*N*C < 2^62.  B = 0: the forward returns WHTMIX_OK without touching anything
+ *               B*N*C <= 2^60.  B = 0: the forward returns WHTMIX_OK without touching anything
  *               (null data pointers are accepted); the backward sets dG to zero (the sum over no
  *               planes) and touches nothing else, so only dgains must be valid.
  *   Alignment   every pointer must be 16-byte aligned.
@@ -171,8 +171,8 @@ WHTMIX_API int whtmix_backward_separable(const void *x, const float *g_t, const 
  * channels, x [T, C] bf16, w [C, C] bf16 stored (out, in) like a linear layer's weight, z [T, C]
  * in out_dtype (WHTMIX_BF16, rounded to nearest even, or WHTMIX_F32); fp32 accumulation.  These
  * are the block's W_in and W_out (Section III-B, Eq. 1 and Eq. 4).  C must be 64, 128 or 256
- * (WHTMIX_ERR_BAD_SHAPE otherwise).  z may be x itself for bf16 output; no other overlap.  16-byte
- * aligned device pointers; T = 0 is a no-op. */
+ * and T*C <= 2^60 (WHTMIX_ERR_BAD_SHAPE otherwise).  z may be x itself for bf16 output; no other
+ * overlap.  16-byte aligned device pointers; T = 0 is a no-op. */
 WHTMIX_API int whtmix_project(const void *x, const void *w, void *z, int64_t T, int64_t C, int out_dtype,
                               void *stream);
 

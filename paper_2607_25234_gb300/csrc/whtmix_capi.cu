@@ -77,7 +77,9 @@ int check_shape(int64_t B, int64_t N, int64_t C, int dtype, int* m) {
   if (!is_pow2(N) || !is_pow2(C)) return WHTMIX_ERR_BAD_SHAPE;
   const int mm = ilog2_pow2(N) + ilog2_pow2(C);
   if (mm > MAX_PLANE_BITS) return WHTMIX_ERR_BAD_SHAPE;
-  if (B > (int64_t{1} << (62 - mm))) return WHTMIX_ERR_BAD_SHAPE;
+  // B*N*C <= 2^60, so that every byte count of the call (up to three padded copies of the batch
+  // at 4 bytes an element) stays far below 2^64
+  if (B > (int64_t{1} << (60 - mm))) return WHTMIX_ERR_BAD_SHAPE;
   *m = mm;
   return WHTMIX_OK;
 }
@@ -688,6 +690,7 @@ int whtmix_backward_separable(const void* x, const float* g_t, const float* g_c,
 int whtmix_project(const void* x, const void* w, void* z, int64_t T, int64_t C, int out_dtype, void* stream_v) {
   if (T < 0 || C < 1) return WHTMIX_ERR_INVALID_ARG;
   if (C != 64 && C != 128 && C != 256) return WHTMIX_ERR_BAD_SHAPE;
+  if (T > (int64_t{1} << 60) / C) return WHTMIX_ERR_BAD_SHAPE;  // T*C <= 2^60: byte counts stay below 2^64
   if (out_dtype != WHTMIX_F32 && out_dtype != WHTMIX_BF16) return WHTMIX_ERR_BAD_DTYPE;
   if (T == 0) return WHTMIX_OK;
   if (!x || !w || !z) return WHTMIX_ERR_INVALID_ARG;

@@ -96,7 +96,7 @@ extern "C" WHTMIX_API int whtmix_forward_noalloc(const void* x, const void* gain
   if (!pow2(N) || !pow2(C)) return WHTMIX_ERR_BAD_SHAPE;
   int m = 0;
   while ((int64_t{1} << m) < N * C) ++m;
-  if (m > MAX_PLANE_BITS || B > (int64_t{1} << (62 - m))) return WHTMIX_ERR_BAD_SHAPE;
+  if (m > MAX_PLANE_BITS || B > (int64_t{1} << (60 - m))) return WHTMIX_ERR_BAD_SHAPE;
   const size_t plane_ws = (size_t{1} << m) * 4;
   if (m > TILE_BITS && plane_ws > WHTMIX_NOALLOC_DATA_BYTES) return WHTMIX_ERR_WORKSPACE;
   if (B == 0) return WHTMIX_OK;
