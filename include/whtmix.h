@@ -42,8 +42,10 @@
  *               nothing.  Faults of the device code surface at the caller's next synchronisation.
  *   Ownership   the caller owns every pointer it passes.  The plain calls keep a workspace per
  *               (device, stream), allocated stream-ordered on first use and grown on demand;
- *               whtmix_release_workspaces() frees them.  The _ex calls use the caller's workspace
- *               instead and allocate nothing.
+ *               whtmix_release_workspaces() frees them.  The cache is keyed by the stream's
+ *               handle, so call it before destroying a stream that plain calls used (a stream
+ *               created later may receive the same handle).  The _ex calls use the caller's
+ *               workspace instead and allocate nothing.
  *   Threads     calls on different streams may run concurrently from different host threads.
  *               Two calls that share a workspace (same stream, or the same _ex buffer) must be
  *               ordered by that stream.
