@@ -332,10 +332,13 @@ def plan(N: int, C: int) -> int:
 
 
 def pad_tokens(x: torch.Tensor, n_pad: int | None = None) -> torch.Tensor:
-    """Zero-pads the token axis (dim -2) to the next power of two, as the paper does before H_N
-    (Section III-B).  Crop the mixer's output back with ``y[..., :n, :]``."""
+    """Zero-pads the token axis (dim -2) to ``n_pad`` tokens (default: the next power of two, at
+    least 1), as the paper does before H_N (Section III-B).  Crop the mixer's output back with
+    ``y[..., :n, :]``."""
     n = x.shape[-2]
-    target = n_pad or (1 << (n - 1).bit_length())
+    target = (1 << max(n - 1, 0).bit_length()) if n_pad is None else n_pad
+    if target < max(n, 1) or target & (target - 1):
+        raise ValueError(f"n_pad must be a power of two >= the {n} tokens of x, got {target}")
     if target == n:
         return x.contiguous()
     pad = torch.zeros(*x.shape[:-2], target - n, x.shape[-1], dtype=x.dtype, device=x.device)

@@ -257,3 +257,21 @@ def test_binding_refuses_cpu_tensors_and_malformed_outputs(monkeypatch):
         whtmix._out(torch.zeros(2, 3), (2, 3), torch.bfloat16, dev, "dx")
     with pytest.raises(ValueError, match="CUDA tensor"):
         whtmix._out(torch.zeros(2, 3), (2, 3), torch.float32, dev, "out")
+
+
+def test_pad_tokens_helper():
+    """whtmix.pad_tokens is plain tensor bookkeeping (no mixer arithmetic): zero rows appended on
+    the token axis up to the next power of two, the stored rows unchanged."""
+    import torch
+    x = torch.arange(2 * 5 * 3, dtype=torch.float32).reshape(2, 5, 3)
+    p = whtmix.pad_tokens(x)
+    assert p.shape == (2, 8, 3) and p.is_contiguous()
+    assert torch.equal(p[:, :5], x) and torch.count_nonzero(p[:, 5:]) == 0
+    assert whtmix.pad_tokens(x, 16).shape == (2, 16, 3)
+    assert whtmix.pad_tokens(x[0]).shape == (8, 3)                     # a single [N, C] plane
+    assert torch.equal(whtmix.pad_tokens(x[:, :4]), x[:, :4])          # already a power of two
+    assert whtmix.pad_tokens(torch.zeros(2, 0, 3)).shape == (2, 1, 3)  # no tokens: one zero row
+    assert whtmix.pad_tokens(torch.zeros(2, 64800, 1)).shape == (2, 65536, 1)
+    for bad in (4, 12):
+        with pytest.raises(ValueError):
+            whtmix.pad_tokens(x, bad)
