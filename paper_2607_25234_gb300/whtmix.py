@@ -93,11 +93,13 @@ def _check(rc: int, what: str):
 def _call(what: str, device: torch.device, stream, fn, *args) -> None:
     """Runs one entry point with ``device`` current, on ``stream`` (default: the device's current
     stream, appended as the last argument); raises WhtmixError on a nonzero status."""
-    with torch.cuda.device(device):
-        s = stream if stream is not None else torch.cuda.current_stream(device)
-        if s.device != device:
-            raise ValueError(f"stream is on {s.device}, the tensors on {device}")
-        _check(fn(*args, int(s.cuda_stream)), what)
+    if device.index != torch.cuda.current_device():
+        with torch.cuda.device(device):
+            return _call(what, device, stream, fn, *args)
+    s = stream if stream is not None else torch.cuda.current_stream(device)
+    if s.device != device:
+        raise ValueError(f"stream is on {s.device}, the tensors on {device}")
+    _check(fn(*args, int(s.cuda_stream)), what)
 
 
 def _on_device(t: torch.Tensor, device: torch.device, name: str) -> None:
