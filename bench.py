@@ -182,11 +182,39 @@ class ClockSampler:
                 "samples": len(inside), "window": window}
 
 
-def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
+def host_cpu():
+    """(usable cores, CPU model) of the host the bench runs on."""
+    try:
+        cores = len(os.sched_getaffinity(0))
+    except Exception:
+        cores = os.cpu_count() or 1
+    model = ""
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    if not model:
+        try:
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for line in out.splitlines():
+                if line.strip().lower().startswith("model name"):
+                    model = line.split(":", 1)[1].strip()
+                    break
+        except Exception:
+            pass
+    return cores, model or "unknown"
+
+
+def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int, threads: int = 1):
     """Median wall time of the CPU oracle on one [n_tokens, C] plane of the workload: the forward,
-    plus the backward for a training-step workload."""
+    plus the backward for a training-step workload, with `threads` OpenMP threads (the results
+    are bit-identical to one thread's)."""
     import numpy as np
     import oracle
+    oracle.set_threads(threads)
     d = inputs.make_inputs(1, n_tokens, w.C, w.dtype, seed=0,
                            n_valid=None if w.n_valid is None else min(w.n_valid, n_tokens), with_dy=w.backward)
     x = inputs.as_float64(d["x"], w.dtype)
@@ -207,6 +235,7 @@ def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int):
         if dy is not None:
             oracle.backward(x, g, dy)
         times.append(time.perf_counter() - t)
+    oracle.set_threads(1)
     return statistics.median(times), times
 
 
@@ -219,7 +248,8 @@ def reference_arm(args, w):
         return
     import numpy as np
     import oracle
-    t_full, _ = oracle_time_plane(w, w.N, 1)
+    cores, model = host_cpu()
+    t_full, _ = oracle_time_plane(w, w.N, 1, cores)
     budget = 180.0
     n = w.N
     while n > 64 and (args.steps + args.warmup) * t_full * n / w.N > budget:
@@ -235,21 +265,25 @@ def reference_arm(args, w):
         run = lambda: oracle.forward_separable(x, g_t, g_c)
     else:
         run = lambda: oracle.forward(x, g)
+    threads = oracle.set_threads(cores)
     for _ in range(args.warmup):
         run()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         run()
     el = time.perf_counter() - t0
+    oracle.set_threads(1)
     value = args.steps * n / el
-    sample = f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s)"
+    sample = (f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s), "
+              f"float64 oracle on {threads} OpenMP threads, CPU {model}")
     metric = "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
     line = {"impl": "reference", "metric": metric, "value": value, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * el / max(args.steps, 1), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": sample,
+                             "cpu_model": model},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -516,17 +550,26 @@ def ours(args, w):
 
     cpu = None
     if not args.no_cpu_baseline:
-        t_med, times = oracle_time_plane(w, w.N, 1 if w.backward else 3)
-        cpu = {"value": w.B * w.N / (t_med * w.B), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+        # the oracle as it stands on the host: all usable cores (OpenMP over rows, column blocks and
+        # elements, bit-identical to one thread) and, beside it, one thread
+        cores, model = host_cpu()
+        reps = 1 if w.backward else 3
+        t_all, times_all = oracle_time_plane(w, w.N, reps, cores)
+        t_one, times_one = oracle_time_plane(w, w.N, reps, 1)
+        what = f"float64 oracle{' forward + backward' if w.backward else ''}"
+        cpu = {"value": w.N / t_all, "unit": "tokens/s", "cores": cores, "kind": "oracle", "cpu_model": model,
                "sample": f"one full [{w.N},{w.C}] plane of the workload (B={w.B} planes would take "
-                         f"{w.B * t_med:.2f} s), float64 oracle{' forward + backward' if w.backward else ''}, "
-                         f"median of {len(times)} run(s): "
-                         + ", ".join(f"{t:.2f}" for t in times) + " s"}
+                         f"{w.B * t_all:.2f} s), {what} on {cores} OpenMP threads, median of {len(times_all)} "
+                         f"run(s): " + ", ".join(f"{t:.3f}" for t in times_all) + " s",
+               "single_thread": {"value": w.N / t_one, "unit": "tokens/s", "cores": 1,
+                                 "sample": f"the same plane on one thread, median of {len(times_one)} run(s): "
+                                           + ", ".join(f"{t:.3f}" for t in times_one) + " s"}}
 
     metric = "WHTMix fwd+bwd tokens/s" if w.backward else "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
     line = {"metric": metric, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "i32" if w.dtype == "i32" else "f32",
+            "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
                        "f32" if w.dtype != "i32" else "i32", "gains": w.gains, "stored_tokens": nv,
                        "parallelism": f"replicas{world}",

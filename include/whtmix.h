@@ -117,17 +117,20 @@ WHTMIX_API int whtmix_backward_ex(const void *x, const void *gains, const void *
 /* Forward that allocates no device memory, for callers that may not allocate while they run:
  * a process whose device memory is owned up front by an outside allocator or framework, a
  * real-time loop where an allocation could stall or fail at the wrong moment, a plugin handed
- * only its input and output buffers.  The paper has no counterpart; this is a deployment variant
- * of whtmix_forward with the same arguments and results.
- * Scratch: the three-phase forward keeps its intermediate planes in a fixed device array of
- * 16 MiB + 256 B defined by the library; every GPU that loads the library holds it until the
+ * only its input and output buffers.  The paper has no counterpart.  Same arguments as
+ * whtmix_forward, and the same kernels for the shape (plane groups limited to the scratch below),
+ * so the results are those of whtmix_forward bit for bit.
+ * Scratch: the kernels keep their barrier header and intermediate planes in a fixed device array
+ * of 16 MiB + 256 B defined by the library; every GPU that loads the library holds it until the
  * process exits.  Limit: planes of N*C <= 2^13 elements need no scratch; larger planes need
  * N*C <= 2^22 (4 Mi fp32 elements), else the call returns WHTMIX_ERR_WORKSPACE and enqueues
- * nothing.  The first call on each device looks up the array's device address with a CUDA
- * runtime call; make that first call before any stream capture.  Each call for N*C > 2^13
- * enqueues a 256-byte memset of the array's barrier header and one kernel.  All calls share the
- * array, which keeps the previous call's contents: calls whose kernels can overlap on the GPU
- * (different streams, or different host threads) race on it -- order them on one stream. */
+ * nothing.  B = 0 is a no-op.  The first call on each device looks up the array's device address
+ * with a CUDA runtime call; make that first call before any stream capture.  A call enqueues two
+ * 4-byte memsets (the barrier's arrival counts) and one kernel.  All calls share the array, which
+ * keeps the previous call's contents: calls whose kernels can overlap on the GPU (different
+ * streams, or different host threads) race on it -- order them on one stream.  A bounded
+ * device-wide wait that gives up sets the array's error word, which stays set (later calls keep
+ * it) until whtmix_sync reports it as WHTMIX_ERR_TIMEOUT and clears it. */
 WHTMIX_API int whtmix_forward_noalloc(const void *x, const void *gains, void *y, int64_t B, int64_t N,
                                       int64_t C, int dtype, void *stream);
 
@@ -191,7 +194,10 @@ WHTMIX_API int whtmix_block_forward(const void *x, const void *w_in, const void 
 /* Synchronises `stream` and reports device-side failures of the calls enqueued on it since the
  * previous whtmix_sync: WHTMIX_ERR_TIMEOUT if a bounded device-wide wait gave up (the library
  * then resets that workspace's barrier), WHTMIX_ERR_CUDA if the synchronisation itself failed,
- * WHTMIX_OK otherwise.  Only the library-managed workspaces of `stream` are checked. */
+ * WHTMIX_OK otherwise.  Checked: the library-managed workspace of `stream` and, on the current
+ * device, the fixed scratch of whtmix_forward_noalloc (pass the stream those calls used, so that
+ * they have finished).  Caller-owned _ex workspaces are the caller's to read (error word at byte
+ * offset 8). */
 WHTMIX_API int whtmix_sync(void *stream);
 
 /* Frees every library-managed workspace on the current device (synchronises the device). */

@@ -34,7 +34,7 @@ def build(force: bool = False) -> str:
     os.makedirs(_BUILD, exist_ok=True)
     if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
         tmp = _LIB_PATH + f".tmp{os.getpid()}"
-        subprocess.run(["gcc", "-std=c11", "-O2", "-fno-fast-math", "-ffp-contract=off", "-fPIC",
+        subprocess.run(["gcc", "-std=c11", "-O2", "-fno-fast-math", "-ffp-contract=off", "-fopenmp", "-fPIC",
                         "-shared", "-o", tmp, _SRC], check=True)
         os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
@@ -57,6 +57,8 @@ def _load():
             for name in ("oracle_wht2d_f64", "oracle_forward_f64", "oracle_forward_u32",
                          "oracle_backward_f64", "oracle_backward_u32"):
                 getattr(lib, name).restype = ctypes.c_int
+            lib.oracle_set_threads.argtypes = [ctypes.c_int]
+            lib.oracle_set_threads.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -76,6 +78,13 @@ def _shape3(x: np.ndarray):
 def _check(rc: int):
     if rc != 0:
         raise ValueError(f"oracle error {rc} (N and C must be powers of two)")
+
+
+def set_threads(k: int) -> int:
+    """Threads for the float64 calls that follow (1, the default: single-threaded).  Only the timed
+    all-core CPU baseline uses more; the results are bit-identical either way.  Returns the count
+    in effect."""
+    return _load().oracle_set_threads(int(k))
 
 
 def fwht(v: np.ndarray) -> np.ndarray:

@@ -27,10 +27,30 @@
  * Layout: X, Y, dY, dX are row-major [B, N, C] (c fastest); G and dG are row-major [N, C].
  * N and C must be powers of two (the paper zero-pads the token axis to the next power of two
  * before the transform; padding is the caller's job here).
+ *
+ * Threads: single-threaded unless oracle_set_threads(k > 1) is called, which only the timed
+ * all-core CPU baseline does.  The threaded mode splits work whose pieces are independent -- the
+ * token rows of a row transform, blocks of channel columns of a column transform, the elements
+ * of the gain step -- so every element goes through exactly the same additions in the same order
+ * and the results are bit-identical to the single-threaded ones.
  */
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+
+static int g_threads = 1;
+
+/* Number of OpenMP threads the next calls use (1: the plain single-threaded loops).  Returns the
+ * count in effect (always 1 when built without OpenMP). */
+int oracle_set_threads(int k) {
+#ifdef _OPENMP
+    g_threads = k < 1 ? 1 : k;
+#else
+    (void)k;
+    g_threads = 1;
+#endif
+    return g_threads;
+}
 
 static int is_pow2(int64_t n) { return n > 0 && (n & (n - 1)) == 0; }
 
@@ -86,11 +106,40 @@ static void fwht_columns_u32(uint32_t *a, int64_t N, int64_t C) {
             }
 }
 
+/* Threaded column transform: each thread takes whole blocks of 8 adjacent channel columns (one
+ * 64-byte line of doubles per row) through all the stages; a column sees the same butterflies in
+ * the same order as in fwht_columns_f64. */
+static void fwht_columns_par_f64(double *a, int64_t N, int64_t C) {
+    const int64_t nblk = (C + 7) / 8;
+#pragma omp parallel for num_threads(g_threads) schedule(static)
+    for (int64_t blk = 0; blk < nblk; ++blk) {
+        const int64_t c0 = 8 * blk, c1 = c0 + 8 < C ? c0 + 8 : C;
+        for (int64_t h = 1; h < N; h *= 2)
+            for (int64_t i = 0; i < N; i += 2 * h)
+                for (int64_t j = i; j < i + h; ++j) {
+                    double *r0 = a + j * C, *r1 = a + (j + h) * C;
+                    for (int64_t c = c0; c < c1; ++c) {
+                        double p = r0[c], q = r1[c];
+                        r0[c] = p + q;
+                        r1[c] = p - q;
+                    }
+                }
+    }
+}
+
+static void fwht_rows_f64(double *a, int64_t N, int64_t C) {
+#pragma omp parallel for num_threads(g_threads) schedule(static) if (g_threads > 1)
+    for (int64_t n = 0; n < N; ++n) oracle_fwht_f64(a + n * C, C, 1);
+}
+
 /* A <- H_N A H_C: the channel transform on every token row (Eq. 2's H_C), then the token
  * transform on every channel column (Eq. 3's H_N). */
 static void wht2d_f64(double *a, int64_t N, int64_t C) {
-    for (int64_t n = 0; n < N; ++n) oracle_fwht_f64(a + n * C, C, 1);
-    fwht_columns_f64(a, N, C);
+    fwht_rows_f64(a, N, C);
+    if (g_threads > 1)
+        fwht_columns_par_f64(a, N, C);
+    else
+        fwht_columns_f64(a, N, C);
 }
 
 static void wht2d_u32(uint32_t *a, int64_t N, int64_t C) {
@@ -101,8 +150,11 @@ static void wht2d_u32(uint32_t *a, int64_t N, int64_t C) {
 /* Inverse order of the same two transforms (columns, then rows); H is its own inverse up to
  * the scale, so only the order differs. */
 static void wht2d_inv_f64(double *a, int64_t N, int64_t C) {
-    fwht_columns_f64(a, N, C);
-    for (int64_t n = 0; n < N; ++n) oracle_fwht_f64(a + n * C, C, 1);
+    if (g_threads > 1)
+        fwht_columns_par_f64(a, N, C);
+    else
+        fwht_columns_f64(a, N, C);
+    fwht_rows_f64(a, N, C);
 }
 
 static void wht2d_inv_u32(uint32_t *a, int64_t N, int64_t C) {
@@ -128,6 +180,7 @@ int oracle_forward_f64(const double *x, const double *g, double *y, int64_t B, i
         double *a = y + b * L;
         memcpy(a, x + b * L, (size_t)L * sizeof(double));
         wht2d_f64(a, N, C);                                   /* (i), (ii)  */
+#pragma omp parallel for num_threads(g_threads) schedule(static) if (g_threads > 1)
         for (int64_t i = 0; i < L; ++i) a[i] = a[i] * g[i] * inv_l; /* (iii) gain and 1/(NC) */
         wht2d_inv_f64(a, N, C);                               /* (iv), (v)  */
     }
@@ -163,6 +216,7 @@ int oracle_backward_f64(const double *x, const double *g, const double *dy, doub
         memcpy(v, dy + b * L, (size_t)L * sizeof(double));
         wht2d_f64(u, N, C);                                   /* H X_b H   */
         wht2d_f64(v, N, C);                                   /* H dY_b H  */
+#pragma omp parallel for num_threads(g_threads) schedule(static) if (g_threads > 1)
         for (int64_t i = 0; i < L; ++i) {
             dg[i] += u[i] * v[i] * inv_l;                     /* b ascending */
             v[i] = v[i] * g[i] * inv_l;

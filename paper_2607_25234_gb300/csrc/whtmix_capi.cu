@@ -84,18 +84,19 @@ int check_shape(int64_t B, int64_t N, int64_t C, int dtype, int* m) {
   return WHTMIX_OK;
 }
 
-int planes_per_group(int64_t B, int m, int backward) {
+// Planes per group: as many as fit in `target` bytes of plane-group workspace (at least one).
+int planes_per_group(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES) {
   if (B == 0) return 1;
   const size_t per = (size_t{1} << m) * 4 * (backward && m > TILE_BITS ? 2 : 1);
-  int64_t gp = static_cast<int64_t>(WS_TARGET_BYTES / per);
+  int64_t gp = static_cast<int64_t>(target / per);
   if (gp < 1) gp = 1;
   if (gp > B) gp = B;
   return static_cast<int>(gp);
 }
 
-size_t workspace_bytes(int64_t B, int m, int backward) {
+size_t workspace_bytes(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES) {
   if (m <= TILE_BITS && !backward) return HEADER_BYTES;
-  const int gp = planes_per_group(B, m, backward);
+  const int gp = planes_per_group(B, m, backward, target);
   const size_t per = (size_t{1} << m) * 4 * (backward && m > TILE_BITS ? 2 : 1);
   return HEADER_BYTES + per * static_cast<size_t>(gp);
 }
@@ -372,6 +373,12 @@ struct Call {
   // the mixer block's projections (Eq. 1 and 4), fused into the forward; null for the mixer alone
   const void* w_in = nullptr;
   const void* w_out = nullptr;
+  // bytes of plane-group workspace a group may fill (smaller for a fixed-size scratch)
+  size_t group_target = WS_TARGET_BYTES;
+  // clear the barrier's two arrival counts before the launch, keeping its error word (a fixed
+  // scratch shared by every call: a wait that gave up in an earlier call must not leave counts
+  // behind, and its error stays set until whtmix_sync reports it)
+  bool reset_arrivals = false;
 };
 
 // Workspace layout of a call: the kernel workspace (barrier header + plane group) first, then
@@ -392,7 +399,7 @@ Layout plan_call(const Call& c, int m) {
   const bool fast = c.backward ? use_fast_backward(c.dtype, m) : use_fast_forward(c.dtype, m);
   l.pad_copy = lv < L && !(fast && (lv * es) % 16 == 0);
   l.fast_sep = c.separable && !c.backward && !l.pad_copy && use_fast_separable(c.dtype, m, cbits);
-  l.base = workspace_bytes(c.B, m, c.backward);  // exactly whtmix_workspace_bytes for a plain call
+  l.base = workspace_bytes(c.B, m, c.backward, c.group_target);  // whtmix_workspace_bytes for a plain call
   size_t off = l.base;
   if (c.separable || l.pad_copy) off = align256(off);
   if (l.fast_sep) {
@@ -519,6 +526,12 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
     if (rc != WHTMIX_OK) return rc;
   }
   char* wsb = static_cast<char*>(ws);
+  if (c.reset_arrivals) {
+    GridBarrier* h = static_cast<GridBarrier*>(ws);
+    cudaError_t e0 = cudaMemsetAsync(&h->count, 0, sizeof(h->count), stream);
+    if (e0 == cudaSuccess) e0 = cudaMemsetAsync(&h->count_odd, 0, sizeof(h->count_odd), stream);
+    if (e0 != cudaSuccess) return cuda_fail(e0);
+  }
   const int cbits = ilog2_pow2(c.C);
   Params P{};
   P.x = c.x;
@@ -534,7 +547,7 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
   P.ws = wsb + HEADER_BYTES;
   P.B = c.B;
   P.m = m;
-  P.gp = planes_per_group(c.B, m, c.backward);
+  P.gp = planes_per_group(c.B, m, c.backward, c.group_target);
   P.scale = 1.0f / static_cast<float>(L);
   P.gt = c.gt;
   P.gc = c.gc;
@@ -641,6 +654,21 @@ Call separable_call(bool backward, const void* x, const float* gt, const float* 
 bool use_fused_block(int64_t C, int m) { return C == 128 && m >= 21 && m <= 23; }
 
 }  // namespace
+
+namespace whtmix {
+// The forward of whtmix_forward_noalloc (whtmix_noalloc.cu): whtmix_forward's kernel choice with
+// the fixed scratch as the workspace, plane groups limited to what it holds.  A plane that needs
+// more scratch than that returns WHTMIX_ERR_WORKSPACE; nothing is allocated.
+int forward_in_fixed_scratch(const void* x, const void* gains, void* y, int64_t B, int64_t N, int64_t C, int dtype,
+                             void* scratch, size_t scratch_bytes, void* stream) {
+  Call c = full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype);
+  c.group_target = scratch_bytes - HEADER_BYTES;
+  c.reset_arrivals = true;
+  return run(c, scratch, scratch_bytes, true, stream);
+}
+// Device address of the fixed scratch on device `dev`, or null if no call has set it up there.
+void* noalloc_scratch_of(int dev);
+}  // namespace whtmix
 
 extern "C" {
 
@@ -761,20 +789,26 @@ int whtmix_sync(void* stream_v) {
   int dev = 0;
   e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e);
-  void* ptr = nullptr;
+  void* ptrs[2] = {nullptr, whtmix::noalloc_scratch_of(dev)};
   {
     std::lock_guard<std::mutex> lk(g_mu);
     auto it = g_ws.find({dev, stream});
-    if (it != g_ws.end()) ptr = it->second.ptr;
+    if (it != g_ws.end()) ptrs[0] = it->second.ptr;
   }
-  if (!ptr) return WHTMIX_OK;
-  GridBarrier h;
-  e = cudaMemcpy(&h, ptr, sizeof(h), cudaMemcpyDeviceToHost);
-  if (e != cudaSuccess) return cuda_fail(e);
-  if (h.err == 0) return WHTMIX_OK;
-  e = cudaMemset(ptr, 0, HEADER_BYTES);
-  if (e != cudaSuccess) return cuda_fail(e);
-  return WHTMIX_ERR_TIMEOUT;
+  // the stream's library-managed workspace, then the no-allocation scratch of this device (both
+  // keep a set error word until it is reported here)
+  int rc = WHTMIX_OK;
+  for (void* ptr : ptrs) {
+    if (!ptr) continue;
+    GridBarrier h;
+    e = cudaMemcpy(&h, ptr, sizeof(h), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (h.err == 0) continue;
+    e = cudaMemset(ptr, 0, HEADER_BYTES);
+    if (e != cudaSuccess) return cuda_fail(e);
+    rc = WHTMIX_ERR_TIMEOUT;
+  }
+  return rc;
 }
 
 int whtmix_release_workspaces(void) {

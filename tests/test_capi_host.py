@@ -198,6 +198,20 @@ def test_padded_rejects_invalid_arguments_before_any_device_work(lib):
     assert sfwd(lib, nv=0) == 0
 
 
+def test_noalloc_rejects_invalid_arguments_before_any_device_work(lib):
+    nf = lib.whtmix_forward_noalloc
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 1 << 32, 1 << 32, 0, None) == 2   # N*C = 2^64: no overflow
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 1 << 62, 4, 0, None) == 2
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 65536, 1024, 0, None) == 9      # 2^26: beyond the fixed scratch
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 65536, 128, 1, None) == 9       # 2^23 bf16 (32 MiB of scratch)
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 6, 4, 0, None) == 2
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, -1, 4, 4, 0, None) == 1
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 4, 4, 7, None) == 3
+    assert nf(None, None, None, 0, 4, 4, 0, None) == 0                     # nothing to do
+    if not GPU_PRESENT:
+        assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 4, 4, 0, None) == 8         # valid: stops at the device
+
+
 def test_project_and_block_reject_invalid_arguments_before_any_device_work(lib):
     P = lib.whtmix_project
     assert P(FAKE, 2 * FAKE, 3 * FAKE, 1, 96, 1, None) == 2        # C must be 64, 128 or 256

@@ -359,3 +359,25 @@ def test_normal_generator_moments():
     assert abs(z.mean()) < 5e-3 and abs(z.std() - 1.0) < 5e-3
     d = inputs.make_inputs(1, 65536, 128, "bf16", n_valid=64800)
     assert (d["x"][0, 64800:] == 0).all() and (d["x"][0, :64800] != 0).mean() > 0.99
+
+
+@pytest.mark.parametrize("B,N,C", [(3, 64, 32), (2, 1024, 4), (1, 1, 256), (2, 512, 1), (1, 4096, 64)])
+def test_threaded_oracle_is_bit_identical_to_single_threaded(B, N, C):
+    """The all-core CPU baseline's threaded mode splits only independent work (rows, column
+    blocks, elements), so forward and backward must match the single-threaded oracle bit for bit."""
+    d = inputs.make_inputs(B, N, C, "f32", seed=B + N + C, with_dy=True)
+    x, g, dy = (d[k].astype(np.float64) for k in ("x", "g", "dy"))
+    try:
+        assert oracle.set_threads(1) == 1
+        y1 = oracle.forward(x, g)
+        dx1, dg1 = oracle.backward(x, g, dy)
+        w1 = oracle.wht2d(x)
+        if oracle.set_threads(4) != 4:
+            pytest.skip("oracle built without OpenMP")
+        y4 = oracle.forward(x, g)
+        dx4, dg4 = oracle.backward(x, g, dy)
+        w4 = oracle.wht2d(x)
+    finally:
+        oracle.set_threads(1)
+    for a, b in ((y1, y4), (dx1, dx4), (dg1, dg4), (w1, w4)):
+        np.testing.assert_array_equal(a, b)
