@@ -638,6 +638,93 @@ def sweep(args):
                       "paper_context": "paper (RTX 4090): isolated WHTMix slope 0.25, attention 1.70"}), flush=True)
 
 
+def floor(args):
+    """The memory-only floor of the three-phase forward on the full-image plane (2^23 elements,
+    bf16 X and Y, fp32 G and workspace): bench_floor.cu moves the mixer's data phase by phase (X ->
+    workspace rows, workspace and G columns, workspace rows -> Y) with coalesced 16-byte accesses,
+    the same per-CTA ownership and the same barriers, and computes no butterflies.  Timed like the
+    mixer (K launches back to back, inputs rotating over > 3x L2), with the mixer itself timed
+    beside it on the same buffers; per-phase times come from global-timer stamps of every CTA
+    (phase k ends when its last CTA leaves it).  Prints one JSON line."""
+    import ctypes
+    import numpy as np
+    import torch
+    from paper_2607_25234_gb300 import build, whtmix
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    lib = whtmix.library()
+    flib = ctypes.CDLL(build.FLOOR_LIB)
+    p, i = ctypes.c_void_p, ctypes.c_int
+    flib.whtmix_floor_three_phase.argtypes = [p, p, p, p, p, i, i, p]
+    flib.whtmix_floor_three_phase.restype = ctypes.c_int
+    w = inputs.WORKLOADS[DEFAULT_WORKLOAD]
+    m = (w.N * w.C).bit_length() - 1
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    l2 = getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0) or 132 * 2**20
+    d = inputs.workload_inputs(w, seed=0)
+    x0 = torch.from_numpy(d["x"].view(np.int16)).to(dev).view(torch.bfloat16)
+    g0 = torch.from_numpy(d["g"]).to(dev)
+    set_bytes = 2 * x0.numel() * 2 + g0.numel() * 4
+    nsets = max(2, -(-3 * l2 // set_bytes))
+    xs = [x0] + [x0.clone() for _ in range(nsets - 1)]
+    gs = [g0] + [g0.clone() for _ in range(nsets - 1)]
+    ys = [torch.empty_like(x0) for _ in range(nsets)]
+    ws = torch.zeros(256 + 4 * (1 << m), dtype=torch.uint8, device=dev)
+    KS = 50
+    stamps = torch.zeros(KS, sms, 4, dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    sp = int(stream.cuda_stream)
+
+    def fl(k, st=None):
+        rc = flib.whtmix_floor_three_phase(xs[k % nsets].data_ptr(), gs[k % nsets].data_ptr(), ys[k % nsets].data_ptr(),
+                                           ws.data_ptr(), (st if st is not None else stamps[0]).data_ptr(), m, sms, sp)
+        if rc != 0:
+            raise RuntimeError(f"floor kernel launch failed: cudaError {rc}")
+
+    def mx(k):
+        whtmix.forward(xs[k % nsets], gs[k % nsets], out=ys[k % nsets])
+
+    def timed(f, K):
+        for k in range(max(args.warmup, 3)):
+            f(k)
+        torch.cuda.synchronize(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for k in range(K):
+            f(k)
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        return 1e3 * a.elapsed_time(b) / K
+
+    K = args.steps
+    floor_us = timed(fl, K)
+    mixer_us = timed(mx, K)
+    floor_us2 = timed(fl, K)
+    for k in range(KS):
+        fl(k, stamps[k])
+    torch.cuda.synchronize(dev)
+    whtmix.sync()
+    hdr = ws[:256].view(torch.int32)
+    if hdr[2].item() != 0:
+        raise RuntimeError("floor kernel: a bounded barrier wait gave up")
+    st = stamps.cpu().numpy().astype(np.float64)
+    t0 = st[:, :, 0].min(axis=1)
+    ends = [st[:, :, k].max(axis=1) for k in (1, 2, 3)]
+    ph = [np.median(ends[0] - t0) / 1e3, np.median(ends[1] - ends[0]) / 1e3, np.median(ends[2] - ends[1]) / 1e3]
+    ideal = w.ideal_bytes()
+    peak, peak_kind = measured_peaks()
+    fus = min(floor_us, floor_us2)
+    print(json.dumps({
+        "metric": "three-phase memory-only floor (no butterflies) vs the mixer, full-image plane",
+        "workload": w.name, "steps": K, "floor_us": fus, "floor_us_runs": [floor_us, floor_us2],
+        "mixer_us": mixer_us, "mixer_over_floor": mixer_us / fus,
+        "floor_phases_us": {"phase1_rows_in": ph[0], "phase2_columns_incl_barrier": ph[1],
+                            "phase3_rows_out_incl_barrier": ph[2], "stamped_launches": KS},
+        "bytes": {"hbm_algorithmic": ideal, "l2_workspace": 4 * 4 * (1 << m)},
+        "floor_frac_of_hbm_peak": ideal / (fus * 1e-6) / 1e9 / peak, "peak_gbs": peak, "peak_kind": peak_kind,
+        "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / l2:.1f}x L2)"}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -647,9 +734,14 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=inputs.WORKLOAD_ORDER)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="isolated-mixer latency vs N (batch 1, C=64) instead")
+    ap.add_argument("--floor", action="store_true",
+                    help="memory-only floor of the three-phase forward on the full-image plane instead")
     args = ap.parse_args()
     if args.sweep:
         sweep(args)
+        return
+    if args.floor:
+        floor(args)
         return
     w = inputs.WORKLOADS[args.workload]
     if args.impl == "reference":

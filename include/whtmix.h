@@ -29,7 +29,7 @@
  *               WHTMIX_I32:  X/Y/dY/dX int32, G/dG int32, UNnormalised (no 1/(N C)), every
  *                            operation wraps modulo 2^32 -- the result is exact and independent
  *                            of the order of the butterfly stages.
- *   Shapes      B >= 0, N >= 1 and C >= 1 powers of two, N*C <= 2^26 elements per plane,
+ *   Shapes      B >= 0, N >= 1 and C >= 1 powers of two, N*C <= 2^30 elements per plane,
  *               B*N*C <= 2^60.  B = 0: the forward returns WHTMIX_OK without touching anything
  *               (null data pointers are accepted); the backward sets dG to zero (the sum over no
  *               planes) and touches nothing else, so only dgains must be valid.
@@ -71,7 +71,7 @@ typedef enum { WHTMIX_F32 = 0, WHTMIX_BF16 = 1, WHTMIX_I32 = 2 } whtmix_dtype_t;
 typedef enum {
     WHTMIX_OK = 0,
     WHTMIX_ERR_INVALID_ARG = 1, /* null pointer where data is needed, B < 0, N < 1 or C < 1   */
-    WHTMIX_ERR_BAD_SHAPE = 2,   /* N or C not a power of two, N*C > 2^26, B*N*C too large     */
+    WHTMIX_ERR_BAD_SHAPE = 2,   /* N or C not a power of two, N*C > 2^30, B*N*C too large     */
     WHTMIX_ERR_BAD_DTYPE = 3,   /* dtype not one of whtmix_dtype_t                             */
     WHTMIX_ERR_MISALIGNED = 4,  /* a pointer is not 16-byte aligned                            */
     WHTMIX_ERR_ALIAS = 5,       /* partial overlap between an output and another buffer        */
@@ -84,8 +84,8 @@ typedef enum {
 /* Forward mixer.  Section III-B, Eq. 1-4 (the map between W_in and W_out).
  *   x      [B, N, C] input planes (dtype)            gains  [N, C] G (float32, int32 for I32)
  *   y      [B, N, C] output planes (dtype); may equal x.
- * Returns a whtmix_status_t.  One kernel launch on `stream` (two for some shapes; none when
- * B = 0). */
+ * Returns a whtmix_status_t.  One kernel launch on `stream` (two for some shapes, five per plane
+ * group for planes of more than 2^26 elements; none when B = 0). */
 WHTMIX_API int whtmix_forward(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
                    int dtype, void *stream);
 
@@ -104,10 +104,11 @@ WHTMIX_API int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype
 
 /* Same as whtmix_forward / whtmix_backward with a caller-owned device workspace of at least
  * whtmix_workspace_bytes() bytes, 256-byte aligned.  Its first 256 bytes hold a device-wide
- * barrier (32-bit words: arrival count, generation, error, second arrival count) and must be zero
- * before the first call that uses the buffer (cudaMemset); every call that completes leaves both
- * counts and the error word zero (the generation word keeps advancing, which is harmless).  Calls sharing
- * a workspace must be ordered on one stream. */
+ * barrier (32-bit words 0, 1, 3, 4: arrival counters; word 2: error; word 5: barrier sequence
+ * number) and must be zero before the first call that uses the buffer (cudaMemset), and again
+ * after a call whose wait gave up (non-zero error word); a call that completes leaves the header
+ * in the state the next call continues from.  Calls sharing a workspace must be ordered on one
+ * stream. */
 WHTMIX_API int whtmix_forward_ex(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
                       int dtype, void *workspace, size_t workspace_bytes, void *stream);
 WHTMIX_API int whtmix_backward_ex(const void *x, const void *gains, const void *dy, void *dx, void *dgains,
@@ -210,9 +211,11 @@ WHTMIX_API const char *whtmix_status_string(int status);
 WHTMIX_API int whtmix_last_cuda_error(void);
 
 /* Which kernel plan a shape uses: 1 = one tile per plane group (N*C <= 2^13), 2 = three
- * passes through the workspace (2^13 < N*C <= 2^26); 0 for an invalid shape.  (The fp32 / bf16
- * forward of a 2^14- or 2^15-element plane with full gains, and of a 2^16-element plane in batches of
- * 80 or more, runs one plane per CTA instead, in the SM's tensor memory, without the workspace.) */
+ * passes through the workspace in one launch (2^13 < N*C <= 2^26), 3 = five passes, one launch
+ * each (seven for the backward), through the workspace (2^26 < N*C <= 2^30); 0 for an invalid
+ * shape.  (The fp32 / bf16 forward of a 2^14- or 2^15-element plane with full gains, and of a
+ * 2^16-element plane in batches of 80 or more, runs one plane per CTA instead, in the SM's tensor
+ * memory, without the workspace.) */
 WHTMIX_API int whtmix_plan(int64_t N, int64_t C);
 
 #ifdef __cplusplus

@@ -18,6 +18,9 @@ LIB = os.path.join(LIBDIR, "libwhtmix.so")
 SOURCES = ["whtmix_capi.cu", "whtmix_fast_f32.cu", "whtmix_fast_bf16.cu", "whtmix_fast_sep_f32.cu", "whtmix_block.cu", "whtmix_plane.cu",
            "whtmix_fast_sep_bf16.cu", "whtmix_noalloc.cu", "whtmix_proj.cu"]
 OBJDIR = os.path.join(LIBDIR, "obj")
+# the bench's memory-only floor model of the three-phase forward (bench.py --floor); not the mixer
+FLOOR_SOURCE = "bench_floor.cu"
+FLOOR_LIB = os.path.join(LIBDIR, "libwhtmix_floor.so")
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 
@@ -37,10 +40,13 @@ def _deps() -> list[str]:
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
-        return False
-    t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(f) <= t for f in _deps())
+    for lib in (LIB, FLOOR_LIB):
+        if not os.path.exists(lib):
+            return False
+        t = os.path.getmtime(lib)
+        if not all(os.path.getmtime(f) <= t for f in _deps()):
+            return False
+    return True
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
@@ -53,18 +59,20 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if verbose:
         common += ["-Xptxas", "-v"]
     procs, objs = [], []
-    for src in SOURCES:
+    for src in SOURCES + [FLOOR_SOURCE]:
         obj = os.path.join(OBJDIR, src.replace(".cu", f".{os.getpid()}.o"))
         objs.append(obj)
         procs.append((src, subprocess.Popen(common + ["-c", os.path.join(CSRC, src), "-o", obj])))
     failed = [src for src, p in procs if p.wait() != 0]
     if failed:
         raise RuntimeError(f"nvcc failed for {failed}")
-    tmp = LIB + f".tmp{os.getpid()}"
-    subprocess.run([nvcc(), ARCH, "-shared", "-o", tmp] + objs + ["-lcudart"], check=True)
-    for obj in objs:
+    floor_obj = objs.pop()
+    for lib, lib_objs in ((LIB, objs), (FLOOR_LIB, [floor_obj])):
+        tmp = lib + f".tmp{os.getpid()}"
+        subprocess.run([nvcc(), ARCH, "-shared", "-o", tmp] + lib_objs + ["-lcudart"], check=True)
+        os.replace(tmp, lib)
+    for obj in objs + [floor_obj]:
         os.remove(obj)
-    os.replace(tmp, LIB)
     return LIB
 
 

@@ -1,5 +1,5 @@
 // Fused mixer block (Section III-B, Eq. 1-4) for bf16 planes of 128 channels and 2^21..2^23
-// elements: one persistent cooperative launch (one CTA per SM).
+// elements: one persistent launch (one CTA per SM, all resident; programmatic stream serialisation).
 #include "whtmix_block.cuh"
 #include "whtmix_fast_launch.cuh"
 
@@ -17,7 +17,7 @@ cudaError_t launch(const Params& P, const void* w_in, const void* w_out, int sms
   const __nv_bfloat16* wi = static_cast<const __nv_bfloat16*>(w_in);
   const __nv_bfloat16* wo = static_cast<const __nv_bfloat16*>(w_out);
   void* args[] = {&p, &wi, &wo};
-  return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, SMEM_BYTES, stream);
+  return launch_pdl(k, static_cast<unsigned>(sms), THREADS, SMEM_BYTES, stream, args);
 }
 
 cudaError_t forward_bf16(const Params& P, const void* w_in, const void* w_out, int sms, cudaStream_t stream) {

@@ -311,6 +311,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_block_fast(Params P, const __nv_
                                                             const __nv_bfloat16* __restrict__ w_out) {
   static_assert(Q >= 7 && Q <= 9, "columns of 128 to 512 rows");
   __shared__ int flag;
+  pdl_wait();
   GridSync gsync(P.bar, &flag);
   const int m = R + Q;
   const int worker = threadIdx.x / WORKER, wt = threadIdx.x % WORKER;
@@ -396,6 +397,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_block_fast(Params P, const __nv_
   fast::tmem_fence_before();
   __syncthreads();
   fast::tmem_fence_after();
+  pdl_trigger();
   if (threadIdx.x < 32) fast::tmem_dealloc_512(blk_tmem_slot);
 }
 

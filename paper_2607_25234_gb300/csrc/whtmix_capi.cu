@@ -200,14 +200,78 @@ int launch(K kernel, bool cooperative, int sms, long long max_units, size_t smem
   if (rc != WHTMIX_OK) return rc;
   long long grid = static_cast<long long>(occ) * sms;
   if (max_units < grid) grid = max_units < 1 ? 1 : max_units;
+  // grid <= resident CTAs: with device-wide barriers (plans M and the backward) every CTA is
+  // resident at once
+  (void)cooperative;
   Params p = P;
   void* args[] = {&p};
-  if (cooperative)
-    e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kernel), dim3(static_cast<unsigned>(grid)), dim3(THREADS), args, smem, stream);
-  else
-    e = cudaLaunchKernel(reinterpret_cast<const void*>(kernel), dim3(static_cast<unsigned>(grid)), dim3(THREADS), args, smem, stream);
+  e = launch_pdl(reinterpret_cast<const void*>(kernel), static_cast<unsigned>(grid), THREADS, smem, stream, args);
   if (e != cudaSuccess) return cuda_fail(e);
   return WHTMIX_OK;
+}
+
+// One launch of a plan-L pass kernel (whtmix_kernels.cuh) over `units` tiles: a grid-stride grid of
+// at most the resident CTAs, programmatic stream serialisation, arguments converted to the kernel's
+// parameter types by the typed cudaLaunchKernelEx.
+template <class... KArgs, class... Args>
+int launch_pass(void (*kernel)(KArgs...), int sms, long long units, size_t smem, cudaStream_t stream, Args... args) {
+  int occ = 0;
+  const int rc = occupancy(reinterpret_cast<const void*>(kernel), smem, &occ);
+  if (rc != WHTMIX_OK) return rc;
+  long long grid = static_cast<long long>(occ) * sms;
+  if (units < grid) grid = units < 1 ? 1 : units;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args...);
+  return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+}
+
+// Plan L (2^26 < N*C <= 2^30): per plane group five passes (forward) or seven (backward), one
+// launch each; the high bits [13, m) are split into [13, 13 + k1) and [13 + k1, m).
+template <int D>
+int dispatch_plan_l(bool backward, const Params& P, int sms, cudaStream_t stream) {
+  using A = typename Tr<D>::A;
+  const int m = P.m, kt = m - TILE_BITS, k1 = kt / 2, k2 = kt - k1;
+  const size_t tb = sizeof(A) * TILE;
+  A* wsx = static_cast<A*>(P.ws);
+  A* wsd = wsx + (static_cast<long long>(P.gp) << m);
+  const long long tiles = 1ll << kt;
+  int rc = WHTMIX_OK;
+#define WHTMIX_PASS(...)                         \
+  do {                                          \
+    rc = launch_pass(__VA_ARGS__);              \
+    if (rc != WHTMIX_OK) return rc;             \
+  } while (0)
+  for (long long b0 = 0; b0 < P.B; b0 += P.gp) {
+    const long long nb = P.B - b0 < P.gp ? P.B - b0 : P.gp;
+    const long long units = nb * tiles;
+    if (!backward) {
+      WHTMIX_PASS(k_pass_rows_in<D>, sms, units, tb, stream, P.x, wsx, b0, nb, m);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsx, nb, m, TILE_BITS, k1, P.g, P.scale, 0);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsx, nb, m, TILE_BITS + k1, k2, P.g, P.scale, 1);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsx, nb, m, TILE_BITS, k1, P.g, P.scale, 0);
+      WHTMIX_PASS(k_pass_rows_out<D>, sms, units, tb, stream, static_cast<const A*>(wsx), P.y, b0, nb, m);
+    } else {
+      WHTMIX_PASS(k_pass_rows_in<D>, sms, units, tb, stream, P.x, wsx, b0, nb, m);
+      WHTMIX_PASS(k_pass_rows_in<D>, sms, units, tb, stream, P.dy, wsd, b0, nb, m);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsx, nb, m, TILE_BITS, k1, P.g, P.scale, 0);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsd, nb, m, TILE_BITS, k1, P.g, P.scale, 0);
+      WHTMIX_PASS(k_pass_cols_bwd<D>, sms, tiles, 3 * tb, stream, wsx, wsd, static_cast<A*>(P.dg), nb, m,
+                  TILE_BITS + k1, k2, P.g, P.scale, b0 == 0 ? 1 : 0);
+      WHTMIX_PASS(k_pass_cols<D>, sms, units, tb, stream, wsd, nb, m, TILE_BITS, k1, P.g, P.scale, 0);
+      WHTMIX_PASS(k_pass_rows_out<D>, sms, units, tb, stream, static_cast<const A*>(wsd), P.dx, b0, nb, m);
+    }
+  }
+#undef WHTMIX_PASS
+  return rc;
 }
 
 // The fast forward (whtmix_fast.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^23.
@@ -225,6 +289,7 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
   using A = typename Tr<D>::A;
   const int m = P.m;
   const size_t tile_bytes = sizeof(A) * TILE;
+  if (m > MAX_PLANE_BITS_M) return dispatch_plan_l<D>(backward, P, sms, stream);
   if (!backward) {
     if constexpr (D != DT_I32) {
       if (use_fast_forward(D, m)) {
@@ -375,7 +440,7 @@ struct Call {
   const void* w_out = nullptr;
   // bytes of plane-group workspace a group may fill (smaller for a fixed-size scratch)
   size_t group_target = WS_TARGET_BYTES;
-  // clear the barrier's two arrival counts before the launch, keeping its error word (a fixed
+  // clear the barrier's arrival counts before the launch, keeping its error word (a fixed
   // scratch shared by every call: a wait that gave up in an earlier call must not leave counts
   // behind, and its error stays set until whtmix_sync reports it)
   bool reset_arrivals = false;
@@ -528,8 +593,8 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
   char* wsb = static_cast<char*>(ws);
   if (c.reset_arrivals) {
     GridBarrier* h = static_cast<GridBarrier*>(ws);
-    cudaError_t e0 = cudaMemsetAsync(&h->count, 0, sizeof(h->count), stream);
-    if (e0 == cudaSuccess) e0 = cudaMemsetAsync(&h->count_odd, 0, sizeof(h->count_odd), stream);
+    cudaError_t e0 = cudaMemsetAsync(h->slot01, 0, sizeof(h->slot01), stream);
+    if (e0 == cudaSuccess) e0 = cudaMemsetAsync(h->slot23, 0, sizeof(h->slot23), stream);
     if (e0 != cudaSuccess) return cuda_fail(e0);
   }
   const int cbits = ilog2_pow2(c.C);
@@ -833,7 +898,7 @@ const char* whtmix_status_string(int status) {
   switch (status) {
     case WHTMIX_OK: return "ok";
     case WHTMIX_ERR_INVALID_ARG: return "invalid argument (null pointer, B < 0, N < 1 or C < 1)";
-    case WHTMIX_ERR_BAD_SHAPE: return "bad shape (N and C must be powers of two, N*C <= 2^26)";
+    case WHTMIX_ERR_BAD_SHAPE: return "bad shape (N and C must be powers of two, N*C <= 2^30)";
     case WHTMIX_ERR_BAD_DTYPE: return "bad dtype (expected WHTMIX_F32, WHTMIX_BF16 or WHTMIX_I32)";
     case WHTMIX_ERR_MISALIGNED: return "pointer not 16-byte aligned";
     case WHTMIX_ERR_ALIAS: return "output partially overlaps another buffer";
@@ -850,7 +915,7 @@ int whtmix_last_cuda_error(void) { return g_last_cuda_error; }
 int whtmix_plan(int64_t N, int64_t C) {
   int m = 0;
   if (check_shape(1, N, C, WHTMIX_F32, &m) != WHTMIX_OK) return 0;
-  return m <= TILE_BITS ? 1 : 2;
+  return m <= TILE_BITS ? 1 : m <= MAX_PLANE_BITS_M ? 2 : 3;
 }
 
 }  // extern "C"

@@ -756,7 +756,6 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 10) || (R == 14 && Q == 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
-  GridSync gsync(P.bar, &flag);
   __shared__ uint32_t tmem_slot;
   constexpr bool USE_TMEM = Q >= 8;
   using RW = Row<R>;
@@ -775,6 +774,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     tmem_fence_after();
     tlane = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16);
   }
+  // tensor memory is allocated before the wait: the previous kernel's CTA on this SM has left
+  pdl_wait();
+  GridSync gsync(P.bar, &flag);
   for (long long b0 = 0; b0 < P.B; b0 += P.gp) {
     const long long nb = min(static_cast<long long>(P.gp), P.B - b0);
     const long long rows = nb << Q;
@@ -837,6 +839,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     }
     if (b0 + P.gp < P.B && !gsync()) break;
   }
+  pdl_trigger();
   if constexpr (USE_TMEM) {
     tmem_fence_before();
     __syncthreads();

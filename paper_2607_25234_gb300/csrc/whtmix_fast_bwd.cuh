@@ -146,7 +146,6 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 7) || (R == 14 && Q == 7), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
-  GridSync gsync(P.bar, &flag);
   __shared__ uint32_t tmem_slot;
   constexpr bool USE_TMEM = Q == 7;
   using RW = Row<R>;
@@ -168,6 +167,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
     // lane quarter of this warp; warps w and w + 4 take TMEM columns [0, 128) and [128, 256)
     tcol = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16) + 128u * (threadIdx.x >> 7);
   }
+  // tensor memory is allocated before the wait: the previous kernel's CTA on this SM has left
+  pdl_wait();
+  GridSync gsync(P.bar, &flag);
   const long long L = 1ll << m;
   const long long lb = ((L >> 2) * blockIdx.x / gridDim.x) << 2, le = ((L >> 2) * (blockIdx.x + 1) / gridDim.x) << 2;
   for (long long b0 = 0; b0 < P.B; b0 += P.gp) {
@@ -220,6 +222,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
     }
     if (b0 + P.gp < P.B && !gsync()) break;
   }
+  pdl_trigger();
   if constexpr (USE_TMEM) {
     tmem_fence_before();
     __syncthreads();

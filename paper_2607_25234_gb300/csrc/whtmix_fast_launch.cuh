@@ -39,7 +39,9 @@ inline cudaError_t occupancy_cached(const void* kernel, size_t smem, int* occ) {
 
 // Every variant requests more than half an SM's shared memory, so exactly one CTA runs per SM:
 // two CTAs on one SM would both ask for all 512 TMEM columns, and the second would wait in
-// tcgen05.alloc while the first waits for it at the device-wide barrier.
+// tcgen05.alloc while the first waits for it at the device-wide barrier.  The grid is one CTA per
+// SM, all resident at once; it is launched with programmatic stream serialisation (launch_pdl),
+// which lets its launch and tensor-memory allocation overlap the previous kernel's tail.
 inline cudaError_t launch_persistent(const void* k, const Params& P, int sms, cudaStream_t stream) {
   const size_t smem = SMEM_BYTES;
   int occ = 0;
@@ -48,7 +50,7 @@ inline cudaError_t launch_persistent(const void* k, const Params& P, int sms, cu
   if (occ != 1) return cudaErrorInvalidConfiguration;
   Params p = P;
   void* args[] = {&p};
-  return cudaLaunchCooperativeKernel(k, dim3(static_cast<unsigned>(sms)), dim3(THREADS), args, smem, stream);
+  return launch_pdl(k, static_cast<unsigned>(sms), THREADS, smem, stream, args);
 }
 template <int D, int R, int Q, bool SEP>
 cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {

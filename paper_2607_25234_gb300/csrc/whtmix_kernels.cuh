@@ -16,6 +16,10 @@
 //       phase 2  each column tile (W = 2^(26-m) adjacent columns x 2^(m-13) rows): bits
 //                [13, m) forward, gain, bits [13, m) inverse                       ws -> ws
 //       phase 3  each row tile: bits [0, 13) again                                 ws -> Y
+//   L (26 < m <= 30): the high bits no longer fit one column tile, so they are split in two
+//     groups [13, 13 + k1) and [13 + k1, m) and the transform runs as five passes, one launch
+//     each (the kernel boundary is the barrier): rows, columns over the first group, columns over
+//     the second with the gain in the middle, the first group again, rows again.
 // Inside a tile the data sits in shared memory (XOR-swizzled) and every round loads 2^e <= 32
 // elements per thread into registers, runs e butterfly stages there and stores them back.
 #pragma once
@@ -29,19 +33,38 @@ namespace whtmix {
 constexpr int TILE_BITS = 13;
 constexpr int TILE = 1 << TILE_BITS;
 constexpr int THREADS = 256;
-constexpr int MAX_PLANE_BITS = 2 * TILE_BITS;
+constexpr int MAX_PLANE_BITS_M = 2 * TILE_BITS;  // plan M: one column tile holds the high bits
+constexpr int MAX_PLANE_BITS = 30;               // plan L up to 2^30 elements per plane
 constexpr int ROUND_BITS = 5;
 constexpr unsigned long long BARRIER_TIMEOUT_NS = 1000000000ull;  // 1 s
 
 enum DType { DT_F32 = 0, DT_BF16 = 1, DT_I32 = 2 };
 
-// Device-wide barrier state; lives in the first 256 bytes of the workspace.
+// Host: launch a kernel that begins with pdl_wait() (and ends with pdl_trigger()) with programmatic
+// stream serialisation, so that its launch and prologue overlap the previous kernel's tail.
+inline cudaError_t launch_pdl(const void* kernel, unsigned int grid, unsigned int block, size_t smem,
+                              cudaStream_t stream, void** args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelExC(&cfg, kernel, args);
+}
+
+// Device-wide barrier state; lives in the first 256 bytes of the workspace.  Barriers are numbered
+// on from call to call (seq); barrier k counts its arrivals in slot k mod 4.
 struct GridBarrier {
-  unsigned int count;      // arrivals at a barrier of even generation (back to 0 after it)
-  unsigned int gen;        // generation, bumped by the last arrival
-  unsigned int err;        // non-zero once a wait gave up
-  unsigned int count_odd;  // arrivals at a barrier of odd generation (back to 0 after it)
-  unsigned int pad[60];
+  unsigned int slot01[2];  // words 0, 1: arrival counts of slots 0 and 1
+  unsigned int err;        // word 2: non-zero once a wait gave up
+  unsigned int slot23[2];  // words 3, 4: arrival counts of slots 2 and 3
+  unsigned int seq;        // word 5: number of the next barrier
+  unsigned int pad[58];
 };
 static_assert(sizeof(GridBarrier) == 256, "barrier header is 256 bytes");
 
@@ -176,11 +199,12 @@ struct PlaneMap {  // plan S: tile = consecutive whole planes
   int lmask;
   __device__ __forceinline__ long long operator()(int i) const { return i & lmask; }
 };
-struct ColMap {  // plan M column tile: i = (row << w) | c  ->  (row << 13) + col0 + c
+struct ColMap {  // column tile: i = (row << w) | c  ->  (row << s) + col0 + c (s = 13 in plan M)
   int w;
   long long col0;
+  int s = TILE_BITS;
   __device__ __forceinline__ long long operator()(int i) const {
-    return (static_cast<long long>(i >> w) << TILE_BITS) + col0 + (i & ((1 << w) - 1));
+    return (static_cast<long long>(i >> w) << s) + col0 + (i & ((1 << w) - 1));
   }
 };
 
@@ -258,16 +282,16 @@ template <class A>
 __device__ __forceinline__ void store_ws_contig(const A* tile, A* dst, long long base) {
   for (int i = threadIdx.x; i < TILE; i += THREADS) dst[base + i] = tile[swz(i)];
 }
-// column tile: i = (row << w) | c  <->  base + (row << 13) + c
+// column tile: i = (row << w) | c  <->  base + (row << s) + c (rows of stride 2^s, s = 13 in plan M)
 template <class A>
-__device__ __forceinline__ void load_ws_col(A* tile, const A* src, long long base, int w) {
+__device__ __forceinline__ void load_ws_col(A* tile, const A* src, long long base, int w, int s = TILE_BITS) {
   for (int i = threadIdx.x; i < TILE; i += THREADS)
-    tile[swz(i)] = ld_ws(src, base + (static_cast<long long>(i >> w) << TILE_BITS) + (i & ((1 << w) - 1)));
+    tile[swz(i)] = ld_ws(src, base + (static_cast<long long>(i >> w) << s) + (i & ((1 << w) - 1)));
 }
 template <class A>
-__device__ __forceinline__ void store_ws_col(const A* tile, A* dst, long long base, int w) {
+__device__ __forceinline__ void store_ws_col(const A* tile, A* dst, long long base, int w, int s = TILE_BITS) {
   for (int i = threadIdx.x; i < TILE; i += THREADS)
-    dst[base + (static_cast<long long>(i >> w) << TILE_BITS) + (i & ((1 << w) - 1))] = tile[swz(i)];
+    dst[base + (static_cast<long long>(i >> w) << s) + (i & ((1 << w) - 1))] = tile[swz(i)];
 }
 
 // ---- device-wide barrier with a bounded wait ----
@@ -282,46 +306,70 @@ __device__ __forceinline__ unsigned int ld_acquire(const unsigned int* p) {
   return v;
 }
 
-// Device-wide barrier of a cooperative launch; every CTA calls it the same number of times.
-// Returns false (and sets bar->err) if this CTA gave up after BARRIER_TIMEOUT_NS; the caller
-// then returns.  Thread 0 of each CTA reads the generation word once, at kernel start (it cannot
-// advance before this CTA arrives), and counts the barriers itself afterwards, so an arrival is
-// one fence and one atomic.  Barriers of even and odd generation count arrivals in separate words:
-// the last arrival releases the others first and clears its counter afterwards, off the critical
-// path, since that counter is next used two barriers later, which no CTA reaches before the last
-// arrival has passed the barrier in between.
+__device__ __forceinline__ void st_relaxed(unsigned int* p, unsigned int v) {
+  asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void red_release_add(unsigned int* p, unsigned int v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned int* barrier_slot(GridBarrier* b, unsigned int k) {
+  k &= 3u;
+  return k < 2 ? &b->slot01[k] : &b->slot23[k - 2];
+}
+
+// Programmatic dependent launch.  The kernels are launched with programmatic stream
+// serialisation, so a kernel's CTAs may start (allocate tensor memory, set up shared memory) while
+// the previous kernel in the stream is finishing.  Before touching global memory every such kernel
+// waits (pdl_wait) until that kernel has completed and its writes are visible; when its own work is
+// done it lets the next kernel begin launching (pdl_trigger).  Triggering only at the end measured
+// best: an early trigger slowed a forward/backward pair by ~35 us (512 against 477 us at
+// [16, 8192, 256]) while the late one keeps the gain on back-to-back forwards (44.2 against 47.0 us
+// at [1, 65536, 128]).  Without the launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Device-wide barrier of a persistent grid of at most the resident-CTA count (every CTA becomes
+// resident as SMs free up; kernels that occupied SMs for ever would make the wait run out instead
+// of hanging); every CTA calls it the same number of times.  Returns false (and sets bar->err) if this CTA gave up after BARRIER_TIMEOUT_NS; the
+// caller then returns.
+// Barrier k: thread 0 of each CTA adds one (release) to slot k mod 4 and polls (acquire) until
+// the slot holds gridDim.x -- the arrivals themselves release the waiters, with no second word
+// to publish.  A slot is cleared by CTA 0 once it has passed the barrier after the slot's (every
+// CTA has then left the slot's barrier), which is three barriers before the slot is used again.
+// The barrier number continues from call to call (seq, read once at kernel start and updated by
+// CTA 0 after each barrier; every CTA has read it by the time CTA 0 passes its first barrier), so
+// the slot left full by a call's last barrier is cleared at the next call's first one.  Must be
+// constructed after pdl_wait().
 struct GridSync {
   GridBarrier* bar;
   int* flag;          // shared: thread 0's verdict for the CTA
-  unsigned int gen;   // thread 0: generation of the next barrier
-  __device__ __forceinline__ GridSync(GridBarrier* b, int* f) : bar(b), flag(f), gen(0) {
-    if (threadIdx.x == 0) gen = ld_acquire(&b->gen);
+  unsigned int k;     // thread 0: number of the next barrier
+  __device__ __forceinline__ GridSync(GridBarrier* b, int* f) : bar(b), flag(f), k(0) {
+    if (threadIdx.x == 0) k = ld_acquire(&b->seq);
   }
   __device__ __forceinline__ bool operator()() {
     __syncthreads();
     if (threadIdx.x == 0) {
       int ok = 1;
-      unsigned int* count = (gen & 1u) ? &bar->count_odd : &bar->count;
-      __threadfence();
-      const unsigned int arrived = atomicAdd(count, 1u);
-      if (arrived == gridDim.x - 1) {
-        __threadfence();
-        atomicAdd(&bar->gen, 1u);
-        atomicExch(count, 0u);
-      } else {
-        // Spin on the generation word (no sleep: the wait is ~1 us and a sleep quantum would add
-        // to it); the clock is read once per 256 polls to bound the wait.
-        const unsigned long long t0 = global_ns();
-        for (unsigned int polls = 1; ld_acquire(&bar->gen) == gen; ++polls) {
-          if ((polls & 255u) == 0 && global_ns() - t0 > BARRIER_TIMEOUT_NS) {
-            atomicOr(&bar->err, 1u);
-            ok = 0;
-            break;
-          }
+      unsigned int* c = barrier_slot(bar, k);
+      red_release_add(c, 1u);
+      // Poll without sleeping (the wait is ~1 us and a sleep quantum would add to it); the clock
+      // is read once per 256 polls to bound the wait.
+      const unsigned long long t0 = global_ns();
+      for (unsigned int polls = 1; ld_acquire(c) != gridDim.x; ++polls) {
+        if ((polls & 255u) == 0 && global_ns() - t0 > BARRIER_TIMEOUT_NS) {
+          atomicOr(&bar->err, 1u);
+          ok = 0;
+          break;
         }
       }
-      __threadfence();
-      ++gen;
+      ++k;
+      if (ok && blockIdx.x == 0) {
+        // plain stores: nobody else writes these words now, and the next arrival's release
+        // orders them before any later use of the slot
+        st_relaxed(barrier_slot(bar, k - 2), 0u);  // the slot of the barrier before this one
+        st_relaxed(&bar->seq, k);
+      }
       *flag = ok;
     }
     __syncthreads();
@@ -335,6 +383,7 @@ template <int D>
 __global__ void __launch_bounds__(THREADS) k_forward_s(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();
   A* tA = reinterpret_cast<A*>(smem_raw);
   const int m = P.m;
   const long long ppt = 1ll << (TILE_BITS - m);
@@ -349,6 +398,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_s(Params P) {
     store_contig<D>(tA, P.y, b0 << m, n);
     __syncthreads();
   }
+  pdl_trigger();
 }
 
 // Forward, plan M (cooperative launch: device-wide barriers between phases).
@@ -357,6 +407,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  pdl_wait();
   GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* ws = static_cast<A*>(P.ws);
@@ -397,6 +448,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
     if (b0 + P.gp < P.B && !gsync()) return;
     (void)L;
   }
+  pdl_trigger();
 }
 
 // Backward, plan S: dX per tile, partial products per plane, then dG summed over b ascending.
@@ -405,6 +457,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_s(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  pdl_wait();
   GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* tB = tA + TILE;
@@ -435,6 +488,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_s(Params P) {
     }
     if (b0 + P.gp < P.B && !gsync()) return;
   }
+  pdl_trigger();
 }
 
 // Backward, plan M: phase 1 row tiles of X and dY -> workspaces; phase 2 each column tile loops
@@ -445,6 +499,7 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
   using A = typename Tr<D>::A;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
+  pdl_wait();
   GridSync gsync(P.bar, &flag);
   A* tA = reinterpret_cast<A*>(smem_raw);
   A* tB = tA + TILE;
@@ -497,6 +552,117 @@ __global__ void __launch_bounds__(THREADS) k_backward_m(Params P) {
     }
     if (b0 + P.gp < P.B && !gsync()) return;
   }
+  pdl_trigger();
+}
+
+// ---------------------------------------------------------------------------------------------
+// Plan L passes (26 < m <= 30), each its own launch over nb planes of the group (planes b0 ... of
+// X, Y, dY, dX; planes 0 ... of the workspaces).
+//
+// Row pass in: each row tile (2^13 contiguous elements) of `src` (dtype D), bits [0, 13) -> ws.
+template <int D>
+__global__ void __launch_bounds__(THREADS) k_pass_rows_in(const void* src, typename Tr<D>::A* ws, long long b0,
+                                                          long long nb, int m) {
+  using A = typename Tr<D>::A;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();
+  A* tA = reinterpret_cast<A*>(smem_raw);
+  const int q = m - TILE_BITS;
+  for (long long u = blockIdx.x; u < (nb << q); u += gridDim.x) {
+    const long long b = u >> q, rt = u & ((1ll << q) - 1);
+    load_contig<D>(tA, src, ((b0 + b) << m) + (rt << TILE_BITS), TILE);
+    __syncthreads();
+    xform(tA, 0, TILE_BITS);
+    store_ws_contig(tA, ws, (b << m) + (rt << TILE_BITS));
+    __syncthreads();
+  }
+  pdl_trigger();
+}
+
+// Row pass out: each row tile of ws, bits [0, 13) -> `dst` (dtype D).
+template <int D>
+__global__ void __launch_bounds__(THREADS) k_pass_rows_out(const typename Tr<D>::A* ws, void* dst, long long b0,
+                                                           long long nb, int m) {
+  using A = typename Tr<D>::A;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();
+  A* tA = reinterpret_cast<A*>(smem_raw);
+  const int q = m - TILE_BITS;
+  for (long long u = blockIdx.x; u < (nb << q); u += gridDim.x) {
+    const long long b = u >> q, rt = u & ((1ll << q) - 1);
+    load_ws_contig(tA, ws, (b << m) + (rt << TILE_BITS));
+    __syncthreads();
+    xform(tA, 0, TILE_BITS);
+    store_contig<D>(tA, dst, ((b0 + b) << m) + (rt << TILE_BITS), TILE);
+    __syncthreads();
+  }
+  pdl_trigger();
+}
+
+// A column tile of the bit group [s, s + k) (k + w = 13): 2^w adjacent elements of each of 2^k rows
+// of stride 2^s, i.e. varying bits [0, w) and [s, s + k); tile t fixes bits [w, s) and [s + k, m).
+__device__ __forceinline__ long long col_tile_base(long long t, int w, int s, int k) {
+  return ((t & ((1ll << (s - w)) - 1)) << w) | ((t >> (s - w)) << (s + k));
+}
+
+// Column pass: bits [s, s + k) of every column tile of nb planes of ws, in place; with gain != 0
+// the forward bits, the gain G/L (no scale for int32) and the same bits again.
+template <int D>
+__global__ void __launch_bounds__(THREADS) k_pass_cols(typename Tr<D>::A* ws, long long nb, int m, int s, int k,
+                                                       const void* g, float scale, int gain) {
+  using A = typename Tr<D>::A;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();
+  A* tA = reinterpret_cast<A*>(smem_raw);
+  const int q = m - TILE_BITS, w = TILE_BITS - k;
+  for (long long u = blockIdx.x; u < (nb << q); u += gridDim.x) {
+    const long long b = u >> q, base = col_tile_base(u & ((1ll << q) - 1), w, s, k);
+    load_ws_col(tA, ws, (b << m) + base, w, s);
+    __syncthreads();
+    if (gain)
+      xform_mid_xform(tA, w, TILE_BITS, GainMid<D, ColMap>{g, scale, ColMap{w, base, s}});
+    else
+      xform(tA, w, TILE_BITS);
+    store_ws_col(tA, ws, (b << m) + base, w, s);
+    __syncthreads();
+  }
+  pdl_trigger();
+}
+
+// Backward gain pass: bits [s, s + k) of the X and dY planes of the group; each column tile owns
+// its dG positions and, in ascending b, adds the planes' (W X)(W dY)/L to them (starting from 0
+// for the first group, else from dG), applies the gain to dY and runs dY's bits back.
+template <int D>
+__global__ void __launch_bounds__(THREADS) k_pass_cols_bwd(typename Tr<D>::A* wsx, typename Tr<D>::A* wsd,
+                                                           typename Tr<D>::A* dg, long long nb, int m, int s, int k,
+                                                           const void* g, float scale, int first) {
+  using A = typename Tr<D>::A;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();
+  A* tA = reinterpret_cast<A*>(smem_raw);
+  A* tB = tA + TILE;
+  A* tC = tB + TILE;
+  const int q = m - TILE_BITS, w = TILE_BITS - k;
+  for (long long t = blockIdx.x; t < (1ll << q); t += gridDim.x) {
+    const long long base = col_tile_base(t, w, s, k);
+    if (first) {
+      for (int i = threadIdx.x; i < TILE; i += THREADS) tC[i] = A(0);
+    } else {
+      load_ws_col(tC, dg, base, w, s);
+    }
+    for (long long b = 0; b < nb; ++b) {
+      load_ws_col(tA, wsx, (b << m) + base, w, s);
+      load_ws_col(tB, wsd, (b << m) + base, w, s);
+      __syncthreads();
+      xform(tA, w, TILE_BITS);
+      xform_mid_xform(tB, w, TILE_BITS, BwdMidM<D>{tA, tC, g, scale, ColMap{w, base, s}});
+      store_ws_col(tB, wsd, (b << m) + base, w, s);
+      __syncthreads();
+    }
+    store_ws_col(tC, dg, base, w, s);
+    __syncthreads();
+  }
+  pdl_trigger();
 }
 
 }  // namespace whtmix

@@ -30,8 +30,9 @@ cudaError_t launch_cb(const Params& P, cudaStream_t stream) {
   const void* k = reinterpret_cast<const void*>(k_forward_plane<D, CB>);
   cudaError_t e = prepare(k);
   if (e != cudaSuccess) return e;
-  k_forward_plane<D, CB><<<static_cast<unsigned>(P.B), THREADS, SMEM_BYTES, stream>>>(P);
-  return cudaGetLastError();
+  Params p = P;
+  void* args[] = {&p};
+  return launch_pdl(k, static_cast<unsigned>(P.B), THREADS, SMEM_BYTES, stream, args);
 }
 
 template <int D>

@@ -244,6 +244,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_plane(Params P) {
   fast::tmem_fence_before();
   __syncthreads();
   fast::tmem_fence_after();
+  pdl_wait();  // tensor memory first: the previous kernel's CTA on this SM has left
   // this thread's lane: warps w and w + 4 (thread wt of either worker) share lane wt
   const uint32_t lane_ta = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16);
   if (worker < NR) {
@@ -268,6 +269,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_plane(Params P) {
     fast::row_loc<R, CB>(0, b * NR + r, P.lv, &e0, &lim);
     row_out<D>(lane_ta + row_col(r), buf, P.y, e0, lim, wt, worker);
   }
+  pdl_trigger();
   fast::tmem_fence_before();
   __syncthreads();
   fast::tmem_fence_after();

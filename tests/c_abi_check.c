@@ -32,7 +32,7 @@ int main(void) {
   EXPECT(whtmix_forward(NULL, g, y, 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_INVALID_ARG);
   EXPECT(whtmix_forward(x, g, y, -1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_INVALID_ARG);
   EXPECT(whtmix_forward(x, g, y, 1, 6, 4, WHTMIX_F32, NULL), WHTMIX_ERR_BAD_SHAPE);
-  EXPECT(whtmix_forward(x, g, y, 1, 1 << 20, 1 << 7, WHTMIX_F32, NULL), WHTMIX_ERR_BAD_SHAPE);
+  EXPECT(whtmix_forward(x, g, y, 1, 1 << 24, 1 << 7, WHTMIX_F32, NULL), WHTMIX_ERR_BAD_SHAPE); /* 2^31 */
   EXPECT(whtmix_forward(x, g, y, ((int64_t)1 << 56) + 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_BAD_SHAPE);
   EXPECT(whtmix_forward(x, g, y, 1, 4, 4, 7, NULL), WHTMIX_ERR_BAD_DTYPE);
   EXPECT(whtmix_forward(P(base + 4), g, y, 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_MISALIGNED);
@@ -57,6 +57,7 @@ int main(void) {
   /* plans, workspace sizes and status strings */
   EXPECT(whtmix_plan(256, 32), 1);
   EXPECT(whtmix_plan(256, 64), 2);
+  EXPECT(whtmix_plan(65536, 2048), 3);
   EXPECT(whtmix_plan(3, 4), 0);
   EXPECT(whtmix_workspace_bytes(1, 256, 32, WHTMIX_F32, 0, &bytes), WHTMIX_OK);
   EXPECT((int)bytes, 256);

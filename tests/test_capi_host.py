@@ -49,8 +49,10 @@ def test_status_strings(lib):
 def test_plan_and_workspace_sizes(lib):
     assert lib.whtmix_plan(256, 32) == 1      # 2^13 elements: one tile
     assert lib.whtmix_plan(256, 64) == 2      # 2^14: three phases
-    assert lib.whtmix_plan(65536, 1024) == 2  # 2^26: largest plane
-    assert lib.whtmix_plan(65536, 2048) == 0  # 2^27: too large
+    assert lib.whtmix_plan(65536, 1024) == 2  # 2^26: largest three-phase plane
+    assert lib.whtmix_plan(65536, 2048) == 3  # 2^27: five passes
+    assert lib.whtmix_plan(1 << 16, 1 << 14) == 3  # 2^30: largest plane
+    assert lib.whtmix_plan(1 << 16, 1 << 15) == 0  # 2^31: too large
     assert lib.whtmix_plan(3, 4) == 0
     ws = whtmix.workspace_bytes
     import torch
@@ -90,7 +92,7 @@ def test_rejects_invalid_arguments_before_any_device_work(lib):
     assert fwd(lib, C=0) == 1
     assert fwd(lib, N=6) == 2
     assert fwd(lib, C=12) == 2
-    assert fwd(lib, N=1 << 20, C=1 << 7) == 2
+    assert fwd(lib, N=1 << 24, C=1 << 7) == 2         # 2^31 elements per plane
     assert fwd(lib, B=(1 << 56) + 1) == 2            # B*N*C above 2^60
     assert fwd(lib, N=1 << 13, C=1 << 13, B=(1 << 34) + 1) == 2
     far = 1 << 60                                     # 2^62 bytes of fp32 at 2^60 elements: no wrap
@@ -203,6 +205,8 @@ def test_noalloc_rejects_invalid_arguments_before_any_device_work(lib):
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 1 << 32, 1 << 32, 0, None) == 2   # N*C = 2^64: no overflow
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 1 << 62, 4, 0, None) == 2
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 65536, 1024, 0, None) == 9      # 2^26: beyond the fixed scratch
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 65536, 2048, 0, None) == 9      # 2^27 (five passes): likewise
+    assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 1 << 16, 1 << 15, 0, None) == 2  # 2^31: no plan
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 65536, 128, 1, None) == 9       # 2^23 bf16 (32 MiB of scratch)
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, 1, 6, 4, 0, None) == 2
     assert nf(FAKE, 2 * FAKE, 3 * FAKE, -1, 4, 4, 0, None) == 1

@@ -3,9 +3,9 @@ complete gives up after its bounded wait (about one second), records the error i
 header's error word and returns; the context stays usable and the next call is correct.
 
 The barrier is made to wait forever the way a missing CTA would: the caller-owned workspace of
-the _ex calls starts with its arrival counter far from zero, so no CTA sees itself as the last
-arrival and nothing ever advances the generation word.  Nothing faults, traps or hangs: every
-CTA leaves on its own after the time limit.
+the _ex calls starts with its four arrival counters far from zero, so no counter ever holds
+exactly the grid's CTA count that releases the waiters.  Nothing faults, traps or hangs: every CTA
+leaves on its own after the time limit.
 """
 import time
 
@@ -46,8 +46,8 @@ def test_stuck_barrier_times_out_and_the_context_stays_usable(B, N, C, dtype, ba
     dy = to_dev(d["dy"], dtype) if backward else None
     ws = torch.zeros(whtmix.workspace_bytes(B, N, C, tdt, backward=backward), dtype=torch.uint8, device="cuda")
     header = ws[:256].view(torch.int32)
-    header[0] = STUCK   # arrivals at even-generation barriers
-    header[3] = STUCK   # arrivals at odd-generation barriers
+    for word in (0, 1, 3, 4):   # the four arrival counters (word 2 is the error word)
+        header[word] = STUCK
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     if backward:
