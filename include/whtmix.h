@@ -192,6 +192,22 @@ WHTMIX_API int whtmix_project(const void *x, const void *w, void *z, int64_t T, 
 WHTMIX_API int whtmix_block_forward(const void *x, const void *w_in, const void *gains, const void *w_out, void *y,
                                     int64_t B, int64_t N, int64_t C, int dtype, void *stream);
 
+/* Backward of the whole mixer block (whtmix_block_forward's map, Section III-B, Eq. 1-4) for the
+ * upstream gradient dY of its output: with Z = X W_in^T and M = mix(Z) recomputed in bf16 (the
+ * forward's activations),
+ *     dM = dY W_out,   (dZ, dG) = whtmix_backward at (Z, G, dM),   dX = dZ W_in,
+ *     dW_out = sum over every token t of dY[t]^T M[t],   dW_in = sum over t of dZ[t]^T X[t].
+ *   x, dy, dx [B, N, C] bf16 (dx may be dy itself); w_in, w_out [C, C] bf16 (out, in); gains [N, C]
+ *   fp32; dw_in, dw_out [C, C] fp32 and dgains [N, C] fp32, all three OVERWRITTEN.
+ * dM and dZ are rounded to bf16 (activation gradients); the weight gradients run on the tensor
+ * cores in fp32 and are summed over token chunks in a fixed order, so every output is the same bit
+ * for bit run to run.  dtype must be WHTMIX_BF16; C 64, 128 or 256.  B = 0 sets the three gain and
+ * weight gradients to zero.  About fifteen launches on `stream`; the intermediates live in a second
+ * library-managed workspace of the stream. */
+WHTMIX_API int whtmix_block_backward(const void *x, const void *w_in, const void *gains, const void *w_out,
+                                     const void *dy, void *dx, void *dw_in, void *dgains, void *dw_out, int64_t B,
+                                     int64_t N, int64_t C, int dtype, void *stream);
+
 /* Synchronises `stream` and reports device-side failures of the calls enqueued on it since the
  * previous whtmix_sync: WHTMIX_ERR_TIMEOUT if a bounded device-wide wait gave up (the library
  * then resets that workspace's barrier), WHTMIX_ERR_CUDA if the synchronisation itself failed,

@@ -175,3 +175,26 @@ def block_forward(x: np.ndarray, w_in: np.ndarray, g: np.ndarray, w_out: np.ndar
     x = np.asarray(x, dtype=np.float64)
     z = x @ np.asarray(w_in, dtype=np.float64).T
     return forward(z, np.asarray(g, dtype=np.float64)) @ np.asarray(w_out, dtype=np.float64).T
+
+
+def block_backward(x: np.ndarray, w_in: np.ndarray, g: np.ndarray, w_out: np.ndarray, dy: np.ndarray):
+    """Gradients of the mixer block of Section III-B, Eq. 1-4, Y = mix(X W_in^T) W_out^T, in
+    float64, for the loss <Y, dY>.  By the chain rule through the three linear steps (Z = X W_in^T,
+    M = mix(Z), Y = M W_out^T), with token rows t over every plane:
+        dM = dY W_out,   (dZ, dG) = the mixer's backward at (Z, G, dM),   dX = dZ W_in,
+        dW_out = sum_t dY[t]^T M[t],   dW_in = sum_t dZ[t]^T X[t].
+    Returns (dX, dW_in, dG, dW_out); the weights are (out, in) like a linear layer's."""
+    x = np.asarray(x, dtype=np.float64)
+    w_in = np.asarray(w_in, dtype=np.float64)
+    w_out = np.asarray(w_out, dtype=np.float64)
+    g = np.asarray(g, dtype=np.float64)
+    dy = np.asarray(dy, dtype=np.float64)
+    C = x.shape[-1]
+    z = x @ w_in.T
+    m = forward(z, g)
+    dm = dy @ w_out
+    dz, dg = backward(z, g, dm)
+    dx = dz @ w_in
+    dw_out = dy.reshape(-1, C).T @ m.reshape(-1, C)
+    dw_in = dz.reshape(-1, C).T @ x.reshape(-1, C)
+    return dx, dw_in, dg, dw_out

@@ -57,23 +57,36 @@ __global__ void __launch_bounds__(FT, 1) k_floor_three_phase(FloorArgs A) {
       if (a1 > a0) prefetch_l2(reinterpret_cast<const char*>(A.g) + a0, static_cast<unsigned>(a1 - a0));
     }
   }
+  // Each phase loads a batch of UNR items per thread into registers before storing any of them,
+  // so that UNR loads per thread are in flight (stores and loads could alias as far as the
+  // compiler knows, which would otherwise serialise every item on its load).
+  constexpr int UNR = 8;
   // phase 1: rows [rb, re) of X -> workspace, 8 bf16 (16 bytes) per item
   {
     const long long v0 = rb << (ROWB - 3), v1 = re << (ROWB - 3);
-    const uint4* xs = reinterpret_cast<const uint4*>(A.x);
-    float4* wd = reinterpret_cast<float4*>(A.ws);
-#pragma unroll 8
-    for (long long v = v0 + threadIdx.x; v < v1; v += FT) {
-      const uint4 u = __ldcs(xs + v);
-      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-      float f[8];
+    const uint4* __restrict__ xs = reinterpret_cast<const uint4*>(A.x);
+    float4* __restrict__ wd = reinterpret_cast<float4*>(A.ws);
+    for (long long vb = v0 + threadIdx.x; vb < v1; vb += UNR * FT) {
+      uint4 u[UNR];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        f[2 * i] = __uint_as_float(w[i] << 16);
-        f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+      for (int j = 0; j < UNR; ++j) {
+        const long long v = vb + j * FT;
+        u[j] = v < v1 ? __ldcs(xs + v) : make_uint4(0u, 0u, 0u, 0u);
       }
-      __stcg(wd + 2 * v, make_float4(f[0], f[1], f[2], f[3]));
-      __stcg(wd + 2 * v + 1, make_float4(f[4], f[5], f[6], f[7]));
+#pragma unroll
+      for (int j = 0; j < UNR; ++j) {
+        const long long v = vb + j * FT;
+        if (v >= v1) continue;
+        const uint32_t w[4] = {u[j].x, u[j].y, u[j].z, u[j].w};
+        float f[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          f[2 * i] = __uint_as_float(w[i] << 16);
+          f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+        __stcg(wd + 2 * v, make_float4(f[0], f[1], f[2], f[3]));
+        __stcg(wd + 2 * v + 1, make_float4(f[4], f[5], f[6], f[7]));
+      }
     }
   }
   if (threadIdx.x == 0) st[1] = global_ns();
@@ -84,13 +97,24 @@ __global__ void __launch_bounds__(FT, 1) k_floor_three_phase(FloorArgs A) {
     const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
     const long long nv = (ce - cb) / 4;  // float4 vectors per row in this CTA's range
     const long long items = nv * rows;
-#pragma unroll 8
-    for (long long it = threadIdx.x; it < items; it += FT) {
-      const long long r = it / nv, c = cb + 4 * (it - r * nv);
-      float4* p = reinterpret_cast<float4*>(A.ws + (r << ROWB) + c);
-      const float4 a = __ldcg(p);
-      const float4 gg = __ldg(reinterpret_cast<const float4*>(A.g + (r << ROWB) + c));
-      __stcg(p, make_float4(a.x * gg.x, a.y * gg.y, a.z * gg.z, a.w * gg.w));
+    for (long long ib = threadIdx.x; ib < items; ib += UNR * FT) {
+      float4 a[UNR], gg[UNR];
+      long long off[UNR];
+#pragma unroll
+      for (int j = 0; j < UNR; ++j) {
+        const long long it = ib + j * FT;
+        const long long r = it / nv;
+        off[j] = (r << ROWB) + cb + 4 * (it - r * nv);
+        if (it < items) {
+          a[j] = __ldcg(reinterpret_cast<const float4*>(A.ws + off[j]));
+          gg[j] = __ldg(reinterpret_cast<const float4*>(A.g + off[j]));
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < UNR; ++j)
+        if (ib + j * FT < items)
+          __stcg(reinterpret_cast<float4*>(A.ws + off[j]),
+                 make_float4(a[j].x * gg[j].x, a[j].y * gg[j].y, a[j].z * gg[j].z, a[j].w * gg[j].w));
     }
   }
   if (threadIdx.x == 0) st[2] = global_ns();
@@ -98,19 +122,31 @@ __global__ void __launch_bounds__(FT, 1) k_floor_three_phase(FloorArgs A) {
   // phase 3: rows [rb, re) of the workspace -> Y, 8 elements per item
   {
     const long long v0 = rb << (ROWB - 3), v1 = re << (ROWB - 3);
-    const float4* ws = reinterpret_cast<const float4*>(A.ws);
-    uint4* yd = reinterpret_cast<uint4*>(A.y);
-#pragma unroll 8
-    for (long long v = v0 + threadIdx.x; v < v1; v += FT) {
-      const float4 a = __ldcg(ws + 2 * v), b = __ldcg(ws + 2 * v + 1);
-      const float f[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-      uint32_t w[4];
+    const float4* __restrict__ ws = reinterpret_cast<const float4*>(A.ws);
+    uint4* __restrict__ yd = reinterpret_cast<uint4*>(A.y);
+    for (long long vb = v0 + threadIdx.x; vb < v1; vb += UNR * FT) {
+      float4 a[UNR], b[UNR];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
-        w[i] = *reinterpret_cast<uint32_t*>(&h);
+      for (int j = 0; j < UNR; ++j) {
+        const long long v = vb + j * FT;
+        if (v < v1) {
+          a[j] = __ldcg(ws + 2 * v);
+          b[j] = __ldcg(ws + 2 * v + 1);
+        }
       }
-      __stcs(yd + v, make_uint4(w[0], w[1], w[2], w[3]));
+#pragma unroll
+      for (int j = 0; j < UNR; ++j) {
+        const long long v = vb + j * FT;
+        if (v >= v1) continue;
+        const float f[8] = {a[j].x, a[j].y, a[j].z, a[j].w, b[j].x, b[j].y, b[j].z, b[j].w};
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+          w[i] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        __stcs(yd + v, make_uint4(w[0], w[1], w[2], w[3]));
+      }
     }
   }
   if (threadIdx.x == 0) st[3] = global_ns();

@@ -9,6 +9,7 @@
 #include <cstring>
 #include <map>
 #include <mutex>
+#include <tuple>
 #include <utility>
 
 #include "whtmix.h"
@@ -30,6 +31,13 @@ namespace proj {
 cudaError_t project(const void* x, const void* w, void* z, long long T, int C, bool out_f32, unsigned int* err, int sms,
                     cudaStream_t s);
 }  // namespace proj
+namespace bbwd {
+// whtmix_block_bwd.cu: the block backward's transposes and weight gradients on the tensor cores
+int wgrad_chunks(long long Tp, int sms);
+cudaError_t transpose(const void* in, void* out, long long T, int C, long long Tp, int sms, cudaStream_t stream);
+cudaError_t wgrad(const void* at, const void* bt, float* part, float* out, long long Tp, int C, int sms,
+                  unsigned int* err, cudaStream_t stream);
+}  // namespace bbwd
 }  // namespace whtmix
 
 using namespace whtmix;
@@ -116,6 +124,11 @@ int device_check(int* dev_out, int* sms_out) {
     g_last_cuda_error = static_cast<int>(e);
     return WHTMIX_ERR_NO_DEVICE;
   }
+  // Bind the device's primary context to this host thread (a no-op where it is already current):
+  // a thread that never set a device -- an autograd worker, a fresh thread of the caller -- then
+  // sees the same context as the one that allocated its buffers.
+  e = cudaSetDevice(dev);
+  if (e != cudaSuccess) return cuda_fail(e);
   std::lock_guard<std::mutex> lk(g_mu);
   DevInfo& di = g_dev[dev];
   if (!di.init) {
@@ -132,16 +145,18 @@ int device_check(int* dev_out, int* sms_out) {
   return WHTMIX_OK;
 }
 
-// ---- library-managed workspaces, one per (device, stream) ----
+// ---- library-managed workspaces, one per (device, stream, slot) ----
+// Slot 0 is the kernels' workspace (barrier header + plane group); slot 1 holds the block
+// backward's intermediates, which must survive the slot-0 calls made in between.
 struct WsEntry {
   void* ptr = nullptr;
   size_t bytes = 0;
 };
-std::map<std::pair<int, cudaStream_t>, WsEntry> g_ws;
+std::map<std::tuple<int, cudaStream_t, int>, WsEntry> g_ws;
 
-int cached_workspace(int dev, cudaStream_t stream, size_t need, void** out) {
+int cached_workspace(int dev, cudaStream_t stream, size_t need, void** out, int slot = 0) {
   std::lock_guard<std::mutex> lk(g_mu);
-  WsEntry& w = g_ws[{dev, stream}];
+  WsEntry& w = g_ws[std::make_tuple(dev, stream, slot)];
   if (w.bytes < need) {
     if (w.ptr) {
       cudaError_t e = cudaFreeAsync(w.ptr, stream);
@@ -838,6 +853,108 @@ int whtmix_block_forward(const void* x, const void* w_in, const void* gains, con
   return whtmix_project(y, w_out, y, T, C, WHTMIX_BF16, stream);
 }
 
+int whtmix_block_backward(const void* x, const void* w_in, const void* gains, const void* w_out, const void* dy,
+                          void* dx, void* dw_in, void* dgains, void* dw_out, int64_t B, int64_t N, int64_t C, int dtype,
+                          void* stream_v) {
+  int m = 0;
+  int rc = check_shape(B, N, C, dtype, &m);
+  if (rc != WHTMIX_OK) return rc;
+  if (dtype != WHTMIX_BF16) return WHTMIX_ERR_BAD_DTYPE;
+  if (C != 64 && C != 128 && C != 256) return WHTMIX_ERR_BAD_SHAPE;
+  if (!dw_in || !dgains || !dw_out) return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(dw_in) || !aligned16(dgains) || !aligned16(dw_out)) return WHTMIX_ERR_MISALIGNED;
+  const size_t wgb = static_cast<size_t>(C) * C * 4, gb = static_cast<size_t>(N) * C * 4;
+  if (overlap(dw_in, wgb, dgains, gb) || overlap(dw_in, wgb, dw_out, wgb) || overlap(dgains, gb, dw_out, wgb))
+    return WHTMIX_ERR_ALIAS;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  int dev = 0, sms = 0;
+  if (B == 0) {  // sums over no tokens
+    rc = device_check(&dev, &sms);
+    if (rc != WHTMIX_OK) return rc;
+    cudaError_t e = cudaMemsetAsync(dw_in, 0, wgb, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dgains, 0, gb, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dw_out, 0, wgb, stream);
+    return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
+  }
+  if (!x || !w_in || !gains || !w_out || !dy || !dx) return WHTMIX_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(w_in) || !aligned16(gains) || !aligned16(w_out) || !aligned16(dy) || !aligned16(dx))
+    return WHTMIX_ERR_MISALIGNED;
+  const long long T = B * N;
+  const size_t pb = static_cast<size_t>(T) * C * 2, wb = static_cast<size_t>(C) * C * 2;
+  // dx may be dy itself (dY is consumed before dZ is written there); no other overlap
+  const void* ins[5] = {x, w_in, gains, w_out, dy};
+  const size_t in_bytes[5] = {pb, wb, gb, wb, pb};
+  void* outs[4] = {dx, dw_in, dgains, dw_out};
+  const size_t out_bytes[4] = {pb, wgb, gb, wgb};
+  for (int o = 0; o < 4; ++o) {
+    for (int i = 0; i < 5; ++i)
+      if (!(o == 0 && i == 4 && outs[o] == ins[i]) && overlap(outs[o], out_bytes[o], ins[i], in_bytes[i]))
+        return WHTMIX_ERR_ALIAS;
+    for (int p = o + 1; p < 4; ++p)
+      if (overlap(outs[o], out_bytes[o], outs[p], out_bytes[p])) return WHTMIX_ERR_ALIAS;
+  }
+  rc = device_check(&dev, &sms);
+  if (rc != WHTMIX_OK) return rc;
+  // slot-1 layout: Z, M, dM [T, C] bf16; a transposed weight [C, C] bf16; the two transposed
+  // operands [C, Tp] bf16 of a weight gradient; its per-chunk partials [chunks, C, C] fp32
+  const long long Tp = (T + 63) / 64 * 64;
+  const int chunks = bbwd::wgrad_chunks(Tp, sms);
+  const size_t tb = static_cast<size_t>(C) * Tp * 2;
+  size_t off[8], total = 0;
+  const size_t sizes[7] = {pb, pb, pb, wb, tb, tb, static_cast<size_t>(chunks) * wgb};
+  for (int i = 0; i < 7; ++i) {
+    off[i] = total;
+    total += align256(sizes[i]);
+  }
+  void* w1 = nullptr;
+  rc = cached_workspace(dev, stream, total, &w1, 1);
+  if (rc != WHTMIX_OK) return rc;
+  char* base = static_cast<char*>(w1);
+  void *Z = base + off[0], *M = base + off[1], *dM = base + off[2], *WT = base + off[3];
+  void *At = base + off[4], *Bt = base + off[5];
+  float* part = reinterpret_cast<float*>(base + off[6]);
+  auto err_word = [&](unsigned int** e) -> int {  // the slot-0 header's error word, read by whtmix_sync
+    void* w0 = nullptr;
+    const int r = cached_workspace(dev, stream, HEADER_BYTES, &w0, 0);
+    *e = &static_cast<GridBarrier*>(w0)->err;
+    return r;
+  };
+  unsigned int* err = nullptr;
+  cudaError_t e = cudaSuccess;
+#define WHTMIX_STEP(call)                  \
+  do {                                     \
+    rc = (call);                           \
+    if (rc != WHTMIX_OK) return rc;        \
+  } while (0)
+#define WHTMIX_CUDA_STEP(call)             \
+  do {                                     \
+    e = (call);                            \
+    if (e != cudaSuccess) return cuda_fail(e); \
+  } while (0)
+  // Eq. 1 and the mixer: Z = X W_in^T, M = mix(Z) (bf16 activations, as the forward's)
+  WHTMIX_STEP(whtmix_project(x, w_in, Z, T, C, WHTMIX_BF16, stream));
+  WHTMIX_STEP(run(full_call(false, Z, gains, nullptr, M, nullptr, B, N, N, C, dtype), nullptr, 0, false, stream));
+  // Eq. 4 backward: dM = dY W_out (the projection with W_out^T), dW_out = dY^T M
+  WHTMIX_CUDA_STEP(bbwd::transpose(w_out, WT, C, static_cast<int>(C), C, sms, stream));
+  WHTMIX_STEP(whtmix_project(dy, WT, dM, T, C, WHTMIX_BF16, stream));
+  WHTMIX_CUDA_STEP(bbwd::transpose(dy, At, T, static_cast<int>(C), Tp, sms, stream));
+  WHTMIX_CUDA_STEP(bbwd::transpose(M, Bt, T, static_cast<int>(C), Tp, sms, stream));
+  WHTMIX_STEP(err_word(&err));
+  WHTMIX_CUDA_STEP(bbwd::wgrad(At, Bt, part, static_cast<float*>(dw_out), Tp, static_cast<int>(C), sms, err, stream));
+  // the mixer's backward: dZ (into dx) and dG
+  WHTMIX_STEP(run(full_call(true, Z, gains, dM, dx, dgains, B, N, N, C, dtype), nullptr, 0, false, stream));
+  // Eq. 1 backward: dW_in = dZ^T X, then dX = dZ W_in in place
+  WHTMIX_CUDA_STEP(bbwd::transpose(dx, At, T, static_cast<int>(C), Tp, sms, stream));
+  WHTMIX_CUDA_STEP(bbwd::transpose(x, Bt, T, static_cast<int>(C), Tp, sms, stream));
+  WHTMIX_STEP(err_word(&err));
+  WHTMIX_CUDA_STEP(bbwd::wgrad(At, Bt, part, static_cast<float*>(dw_in), Tp, static_cast<int>(C), sms, err, stream));
+  WHTMIX_CUDA_STEP(bbwd::transpose(w_in, WT, C, static_cast<int>(C), C, sms, stream));
+  WHTMIX_STEP(whtmix_project(dx, WT, dx, T, C, WHTMIX_BF16, stream));
+#undef WHTMIX_STEP
+#undef WHTMIX_CUDA_STEP
+  return WHTMIX_OK;
+}
+
 int whtmix_workspace_bytes(int64_t B, int64_t N, int64_t C, int dtype, int backward, size_t* out_bytes) {
   if (!out_bytes) return WHTMIX_ERR_INVALID_ARG;
   int m = 0;
@@ -857,7 +974,7 @@ int whtmix_sync(void* stream_v) {
   void* ptrs[2] = {nullptr, whtmix::noalloc_scratch_of(dev)};
   {
     std::lock_guard<std::mutex> lk(g_mu);
-    auto it = g_ws.find({dev, stream});
+    auto it = g_ws.find(std::make_tuple(dev, stream, 0));
     if (it != g_ws.end()) ptrs[0] = it->second.ptr;
   }
   // the stream's library-managed workspace, then the no-allocation scratch of this device (both
@@ -884,7 +1001,7 @@ int whtmix_release_workspaces(void) {
   if (e != cudaSuccess) return cuda_fail(e);
   std::lock_guard<std::mutex> lk(g_mu);
   for (auto it = g_ws.begin(); it != g_ws.end();) {
-    if (it->first.first == dev) {
+    if (std::get<0>(it->first) == dev) {
       if (it->second.ptr) cudaFree(it->second.ptr);
       it = g_ws.erase(it);
     } else {

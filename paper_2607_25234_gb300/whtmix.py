@@ -20,8 +20,8 @@ from . import build as _build
 __all__ = ["forward", "backward", "forward_ex", "backward_ex", "forward_noalloc", "forward_separable",
            "backward_separable",
            "forward_padded", "backward_padded", "project", "block_forward",
-           "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
-           "WHTMixSeparableFunction", "pad_tokens", "EXPORTS", "library"]
+           "block_backward", "workspace_bytes", "sync", "plan", "release_workspaces", "WhtmixError", "WHTMixFunction",
+           "WHTMixSeparableFunction", "WHTMixBlockFunction", "pad_tokens", "EXPORTS", "library"]
 
 # status codes and dtype codes of include/whtmix.h
 OK = 0
@@ -35,7 +35,7 @@ EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmi
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
            "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc", "whtmix_forward_separable",
            "whtmix_backward_separable", "whtmix_forward_padded", "whtmix_backward_padded", "whtmix_project",
-           "whtmix_block_forward")
+           "whtmix_block_forward", "whtmix_block_backward")
 
 
 class WhtmixError(RuntimeError):
@@ -75,6 +75,7 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_forward_padded.argtypes = [p, p, p, i64, i64, i64, i64, i, p]
             lib.whtmix_project.argtypes = [p, p, p, i64, i64, i, p]
             lib.whtmix_block_forward.argtypes = [p, p, p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_block_backward.argtypes = [p, p, p, p, p, p, p, p, p, i64, i64, i64, i, p]
             lib.whtmix_backward_padded.argtypes = [p, p, p, p, p, i64, i64, i64, i64, i, p]
             for name in EXPORTS:
                 if name != "whtmix_status_string":
@@ -289,6 +290,28 @@ def block_forward(x: torch.Tensor, w_in: torch.Tensor, g: torch.Tensor, w_out: t
     return y
 
 
+def block_backward(x: torch.Tensor, w_in: torch.Tensor, g: torch.Tensor, w_out: torch.Tensor, dy: torch.Tensor,
+                   dx: torch.Tensor | None = None, dw_in: torch.Tensor | None = None, dg: torch.Tensor | None = None,
+                   dw_out: torch.Tensor | None = None, stream=None):
+    """(dX, dW_in, dG, dW_out) of block_forward for the upstream gradient dy (bf16); the gain and
+    weight gradients are float32."""
+    B, N, C = _check_tensors(x, g, dy)
+    if dy.shape != x.shape or dy.dtype != x.dtype:
+        raise ValueError("dy must match x in shape and dtype")
+    for t in (w_in, w_out):
+        if t.dtype != torch.bfloat16 or tuple(t.shape) != (C, C):
+            raise ValueError(f"w_in and w_out must be bfloat16 [{C}, {C}]")
+        _on_device(t, x.device, "w_in and w_out")
+    dx = _out(dx, x.shape, x.dtype, x.device, "dx")
+    dw_in = _out(dw_in, (C, C), torch.float32, x.device, "dw_in")
+    dg = _out(dg, g.shape, torch.float32, x.device, "dg")
+    dw_out = _out(dw_out, (C, C), torch.float32, x.device, "dw_out")
+    _call("whtmix_block_backward", x.device, stream, library().whtmix_block_backward, x.data_ptr(), w_in.data_ptr(),
+          g.data_ptr(), w_out.data_ptr(), dy.data_ptr(), dx.data_ptr(), dw_in.data_ptr(), dg.data_ptr(),
+          dw_out.data_ptr(), B, N, C, DTYPE_CODE[x.dtype])
+    return dx, dw_in, dg, dw_out
+
+
 def workspace_bytes(B: int, N: int, C: int, dtype: torch.dtype, backward: bool = False) -> int:
     out = ctypes.c_size_t(0)
     _check(library().whtmix_workspace_bytes(B, N, C, DTYPE_CODE[dtype], int(backward), ctypes.byref(out)),
@@ -376,3 +399,20 @@ class WHTMixSeparableFunction(torch.autograd.Function):
     def backward(ctx, dy):
         x, g_t, g_c = ctx.saved_tensors
         return backward_separable(x, g_t, g_c, dy.contiguous())
+
+
+class WHTMixBlockFunction(torch.autograd.Function):
+    """autograd wrapper of the whole block (W_in, mixer, W_out): forward and backward both run in
+    the CUDA library; the weight and gain gradients come back in float32."""
+
+    @staticmethod
+    def forward(ctx, x, w_in, g, w_out):
+        x, w_in, g, w_out = x.contiguous(), w_in.contiguous(), g.contiguous(), w_out.contiguous()
+        ctx.save_for_backward(x, w_in, g, w_out)
+        return block_forward(x, w_in, g, w_out)
+
+    @staticmethod
+    def backward(ctx, dy):
+        x, w_in, g, w_out = ctx.saved_tensors
+        dx, dw_in, dg, dw_out = block_backward(x, w_in, g, w_out, dy.contiguous())
+        return dx, dw_in.to(w_in.dtype), dg, dw_out.to(w_out.dtype)

@@ -127,3 +127,119 @@ def fused(N, C):
     """True where whtmix_block_forward runs one fused launch (Z stays fp32): C = 128, 2^21..2^23."""
     m = (N * C).bit_length() - 1
     return C == 128 and 21 <= m <= 23
+
+
+# ---- the block backward ----
+
+@pytest.mark.parametrize("B,N,C", [(2, 64, 64), (3, 256, 128), (1, 64, 256), (2, 4096, 128), (1, 65536, 128),
+                                   (4, 8192, 256), (3, 32, 64), (5, 16, 128)])
+def test_block_backward_matches_oracle(B, N, C):
+    """whtmix_block_backward against the float64 block gradients.  Two references: the exact map
+    (acceptance: relative L2 <= 1e-2 per plane for dX, as bf16 outputs, and <= 1e-2 for dW_in, dG,
+    dW_out, whose inputs pass through bf16 activations), and the same gradients with Z, M, dM and dZ
+    rounded to bf16 where the library rounds them (then dX is its bf16 rounding up to a few flipped
+    roundings, and dW_in, dG, dW_out agree to 1e-3).  [3, 32, 64] and [5, 16, 128] have 96 and 80
+    tokens, not a multiple of the weight gradients' 64-token tiles."""
+    d = inputs.make_inputs(B, N, C, "bf16", seed=B + N + C + 1, with_dy=True)
+    w_in = (inputs.normal(92 + C, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32)
+    w_out = (inputs.normal(93 + C, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32)
+    x = torch.from_numpy(d["x"].view(np.int16)).cuda().view(torch.bfloat16)
+    dy = torch.from_numpy(d["dy"].view(np.int16)).cuda().view(torch.bfloat16)
+    g = torch.from_numpy(d["g"]).cuda()
+    wi, wo = bf16_dev(w_in), bf16_dev(w_out)
+    outs = [Guarded(x.shape, torch.bfloat16), Guarded((C, C), torch.float32), Guarded((N, C), torch.float32),
+            Guarded((C, C), torch.float32)]
+    whtmix.block_backward(x, wi, g, wo, dy, dx=outs[0].t, dw_in=outs[1].t, dg=outs[2].t, dw_out=outs[3].t)
+    whtmix.sync()
+    for o, name in zip(outs, ("dX", "dW_in", "dG", "dW_out")):
+        o.assert_intact(f"block {name} [{B},{N},{C}]")
+    x64 = inputs.as_float64(d["x"], "bf16")
+    dy64 = inputs.as_float64(d["dy"], "bf16")
+    wi64 = inputs.as_float64(inputs.f32_to_bf16_bits(w_in), "bf16")
+    wo64 = inputs.as_float64(inputs.f32_to_bf16_bits(w_out), "bf16")
+    g64 = d["g"].astype(np.float64)
+    got = [o.t.double().cpu().numpy() for o in outs]
+    # exact map
+    exact = oracle.block_backward(x64, wi64, g64, wo64, dy64)
+    # rounded where the library rounds: Z, M, dM, dZ to bf16
+    zr = bf16_round(x64 @ wi64.T)
+    mr = bf16_round(oracle.forward(zr, g64))
+    dmr = bf16_round(dy64 @ wo64)
+    dz, dg_r = oracle.backward(zr, g64, dmr)
+    dzr = bf16_round(dz)
+    rounded = [dzr @ wi64, dzr.reshape(-1, C).T @ x64.reshape(-1, C), dg_r, dy64.reshape(-1, C).T @ mr.reshape(-1, C)]
+
+    def rel(a, b):
+        return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+    for k, name in enumerate(("dX", "dW_in", "dG", "dW_out")):
+        if k == 0:
+            for b in range(B):
+                assert rel(got[0][b], exact[0][b]) <= 1e-2, f"dX plane {b}: {rel(got[0][b], exact[0][b]):.3e}"
+                assert rel(got[0][b], rounded[0][b]) <= 5e-3, f"dX plane {b} vs rounded: {rel(got[0][b], rounded[0][b]):.3e}"
+        else:
+            assert rel(got[k], exact[k]) <= 1e-2, f"{name}: {rel(got[k], exact[k]):.3e} vs exact"
+            assert rel(got[k], rounded[k]) <= 1e-3, f"{name}: {rel(got[k], rounded[k]):.3e} vs rounded"
+    # dX element-wise: the final rounding plus a flipped dZ rounding (one ulp, 2^-7 |dZ|) through W_in
+    bound = 2.0 ** -8 * np.abs(rounded[0]) + 2.0 ** -7 * (np.abs(dzr) @ np.abs(wi64)) + 1e-5
+    assert (np.abs(got[0] - rounded[0]) <= bound).all(), float(np.max(np.abs(got[0] - rounded[0]) / bound))
+    # bit-reproducible
+    again = whtmix.block_backward(x, wi, g, wo, dy)
+    torch.cuda.synchronize()
+    for a, o in zip(again, outs):
+        assert torch.equal(a, o.t)
+
+
+def test_block_autograd_function():
+    B, N, C = 2, 512, 128
+    d = inputs.make_inputs(B, N, C, "bf16", seed=77, with_dy=True)
+    w_in = (inputs.normal(94, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32)
+    w_out = (inputs.normal(95, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32)
+    x = torch.from_numpy(d["x"].view(np.int16)).cuda().view(torch.bfloat16).requires_grad_(True)
+    g = torch.from_numpy(d["g"]).cuda().requires_grad_(True)
+    wi, wo = bf16_dev(w_in).requires_grad_(True), bf16_dev(w_out).requires_grad_(True)
+    y = whtmix.WHTMixBlockFunction.apply(x, wi, g, wo)
+    dy = torch.from_numpy(d["dy"].view(np.int16)).cuda().view(torch.bfloat16)
+    y.backward(dy)
+    ref = whtmix.block_backward(x.detach(), wi.detach(), g.detach(), wo.detach(), dy)
+    torch.cuda.synchronize()
+    assert torch.equal(x.grad, ref[0]) and torch.equal(g.grad, ref[2])
+    assert torch.equal(wi.grad, ref[1].to(torch.bfloat16)) and torch.equal(wo.grad, ref[3].to(torch.bfloat16))
+
+
+def test_calls_from_a_thread_that_never_set_the_device():
+    """The autograd engine (and any caller) may call from a host thread that never set a device:
+    every entry point binds the device's context itself, so results match the main thread's."""
+    import threading
+    B, N, C = 2, 512, 128
+    d = inputs.make_inputs(B, N, C, "bf16", seed=78, with_dy=True)
+    x = torch.from_numpy(d["x"].view(np.int16)).cuda().view(torch.bfloat16)
+    dy = torch.from_numpy(d["dy"].view(np.int16)).cuda().view(torch.bfloat16)
+    g = torch.from_numpy(d["g"]).cuda()
+    wi = bf16_dev((inputs.normal(96, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32))
+    wo = bf16_dev((inputs.normal(97, C * C) / np.sqrt(C)).reshape(C, C).astype(np.float32))
+    calls = {
+        "forward": lambda: (whtmix.forward(x, g),),
+        "backward": lambda: whtmix.backward(x, g, dy),
+        "project": lambda: (whtmix.project(x.view(-1, C), wi),),
+        "block_forward": lambda: (whtmix.block_forward(x, wi, g, wo),),
+        "block_backward": lambda: whtmix.block_backward(x, wi, g, wo, dy),
+    }
+    for name, f in calls.items():
+        got = {}
+
+        def run():
+            try:
+                got["r"] = f()
+                torch.cuda.synchronize()
+            except Exception as e:  # reported below, in the test's thread
+                got["e"] = e
+
+        t = threading.Thread(target=run)
+        t.start()
+        t.join()
+        assert "e" not in got, f"{name} from a fresh thread: {got.get('e')}"
+        want = f()
+        torch.cuda.synchronize()
+        for a, b in zip(got["r"], want):
+            assert torch.equal(a, b), name

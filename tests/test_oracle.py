@@ -381,3 +381,50 @@ def test_threaded_oracle_is_bit_identical_to_single_threaded(B, N, C):
         oracle.set_threads(1)
     for a, b in ((y1, y4), (dx1, dx4), (dg1, dg4), (w1, w4)):
         np.testing.assert_array_equal(a, b)
+
+
+def test_block_backward_matches_central_differences():
+    """Every gradient of the block (Eq. 1-4) against central differences of <Y, dY> (the block is
+    linear in each argument, so the differences are exact up to rounding)."""
+    rng = np.random.default_rng(5)
+    B, N, C = 2, 4, 8
+    x = rng.standard_normal((B, N, C))
+    w_in = rng.standard_normal((C, C)) / np.sqrt(C)
+    w_out = rng.standard_normal((C, C)) / np.sqrt(C)
+    g = 1.0 + 0.1 * rng.standard_normal((N, C))
+    dy = rng.standard_normal((B, N, C))
+    dx, dw_in, dg, dw_out = oracle.block_backward(x, w_in, g, w_out, dy)
+
+    def loss(x_, wi_, g_, wo_):
+        return float(np.sum(oracle.block_forward(x_, wi_, g_, wo_) * dy))
+
+    h = 1e-3
+    args = [x, w_in, g, w_out]
+    for k, grad in enumerate((dx, dw_in, dg, dw_out)):
+        num = np.zeros_like(grad)
+        for idx in np.ndindex(grad.shape):
+            plus = [a.copy() for a in args]
+            minus = [a.copy() for a in args]
+            plus[k][idx] += h
+            minus[k][idx] -= h
+            num[idx] = (loss(*plus) - loss(*minus)) / (2 * h)
+        np.testing.assert_allclose(grad, num, rtol=1e-7, atol=1e-9, err_msg=f"gradient {k}")
+
+
+def test_block_backward_special_cases():
+    """Identity projections and unit gains make the block the identity, so every input gradient is
+    dY itself and dG is the plain mixer's; a zero upstream gradient gives zero gradients."""
+    rng = np.random.default_rng(6)
+    B, N, C = 3, 8, 4
+    x = rng.standard_normal((B, N, C))
+    dy = rng.standard_normal((B, N, C))
+    eye = np.eye(C)
+    ones = np.ones((N, C))
+    dx, dw_in, dg, dw_out = oracle.block_backward(x, eye, ones, eye, dy)
+    np.testing.assert_allclose(dx, dy, atol=1e-12)
+    np.testing.assert_allclose(dg, oracle.backward(x, ones, dy)[1], atol=1e-12)
+    # with identity weights and unit gains Y = X, so dW_out = sum_t dY^T X = dW_in
+    np.testing.assert_allclose(dw_out, dy.reshape(-1, C).T @ x.reshape(-1, C), atol=1e-12)
+    np.testing.assert_allclose(dw_in, dw_out, atol=1e-12)
+    z = oracle.block_backward(x, eye, ones, eye, np.zeros_like(dy))
+    assert all(np.count_nonzero(a) == 0 for a in z)
