@@ -76,10 +76,10 @@ def kernel_name(w) -> str:
 def backward_kernel_name(w) -> str:
     """The kernel one whtmix_backward call launches for this workload (mirrors the C ABI's dispatch)."""
     m = (w.N * w.C).bit_length() - 1
-    if w.dtype in ("f32", "bf16") and 14 <= m <= 21:
-        r = 14 if m == 21 else 13
+    if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
+        r = 14 if m >= 21 else 13
         return f"k_backward_fast<{w.dtype}, R={r}, Q={m - r}>"
-    return "k_backward_s" if m <= 13 else "k_backward_m"
+    return "k_backward_s" if m <= 13 else "k_backward_m" if m <= 26 else "k_pass_* (five launches per group)"
 
 
 def kernel_source_hash(kernel: str) -> str:

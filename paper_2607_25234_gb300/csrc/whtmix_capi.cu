@@ -294,9 +294,9 @@ bool use_fast_forward(int dtype, int m) {
   return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 23;
 }
 
-// The fast backward (whtmix_fast_bwd.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^21.
+// The fast backward (whtmix_fast_bwd.cuh) covers fp32 / bf16 planes with 2^14 <= N*C <= 2^23.
 bool use_fast_backward(int dtype, int m) {
-  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 21;
+  return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 23;
 }
 
 template <int D>

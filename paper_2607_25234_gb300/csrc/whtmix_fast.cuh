@@ -594,10 +594,16 @@ __device__ __forceinline__ void lane16_swap(float2 (&v)[8][W], int h) {
 //   round B: bits k6..k(et) (and k9 after a half swap between the lanes) forward, gain, back;
 //            each warp half takes k5 = hw
 //   round C: own ET elements, bits k0..k5 again, TMEM -> global
-template <int Q, int R, class GainT>
+// MODE 0 is the forward's column pass.  The backward (Q = 8, 9) runs two more: MODE 1 takes the
+// column bits forward only and stores the transformed column straight from round B (no gain, no
+// round C); MODE 2 is MODE 0 on the dY workspace, and at the gain step also reads the MODE 1
+// result at the same positions of xws, the transformed X column, and replaces it with the product
+// (W X)(W dY) times `scale` (the dG term of the plane).
+template <int Q, int R, class GainT, int MODE = 0>
 __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, float scale, int m, long long u_begin,
-                                              long long u_end, uint32_t tlane) {
+                                              long long u_end, uint32_t tlane, float* xws = nullptr) {
   constexpr bool LANE_BIT = Q == 10;
+  static_assert(MODE == 0 || (!LANE_BIT && !GainT::SEPARABLE), "the backward modes: Q = 8, 9, full gains");
   constexpr int ET_BITS = LANE_BIT ? 8 : Q - 1;        // 8, 7 for Q = 9, 8; 8 for Q = 10
   constexpr int ET = 1 << ET_BITS;
   constexpr int PER_PASS = LANE_BIT ? 64 : 128;        // columns per pass
@@ -673,56 +679,81 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 #pragma unroll
           for (int w = 0; w < W; ++w) bf2(v[t][w], v[t + 4][w]);
       }
+      if constexpr (MODE == 1) {  // the transformed column, rows j and j + 1 of each pair
+        if (active) {
 #pragma unroll
-      for (int s = 0; s < NH; ++s) {
-        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-        // (Q = 10: after the swap, s / 4 is column bit 9 and the warp-half bit is this lane's l4)
-        const long long j0 = LANE_BIT ? s_hw * 2 * ET + l4 * ET + s_local * 64 + 32 * hw + 2 * W * it
-                                      : s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+          for (int s = 0; s < NH; ++s) {
+            const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+            const long long j0 = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
 #pragma unroll
-        for (int w = 0; w < W; ++w) {
-          const long long j = j0 + 2 * w;
-          float2 gg;
-          // (the full gain's loads are written out here: through at() the compiler spills in this loop)
-          if constexpr (GainT::SEPARABLE) gg = gain.rows2(gcol, j);
-          else gg = make_float2(__ldg(gcol.p + (j << R)), __ldg(gcol.p + ((j + 1) << R)));
-          v[s][w] = mul2(v[s][w], mul2(gg, sc));
-        }
-      }
-      if constexpr (LANE_BIT) {
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-#pragma unroll
-          for (int w = 0; w < W; ++w) bf2(v[t][w], v[t + 4][w]);
-        lane16_swap(v, l4);
-      }
-#pragma unroll
-      for (int hh = 1; hh < NH; hh <<= 1)
-#pragma unroll
-        for (int s = 0; s < NH; ++s)
-          if ((s & hh) == 0)
-#pragma unroll
-            for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
-#pragma unroll
-      for (int s = 0; s < NH; ++s) {
-        const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
-        const uint32_t col = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
-#pragma unroll
-        for (int q = 0; q < 2 * W / 16; ++q) {
-          float t[16];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            t[2 * i] = v[s][8 * q + i].x;
-            t[2 * i + 1] = v[s][8 * q + i].y;
+            for (int w = 0; w < W; ++w) {
+              const long long j = j0 + 2 * w;
+              __stcg(colp + (j << R), v[s][w].x);
+              __stcg(colp + ((j + 1) << R), v[s][w].y);
+            }
           }
-          tmem_st16(tlane + col + 16 * q, t);
         }
-      }
+      } else {
+#pragma unroll
+        for (int s = 0; s < NH; ++s) {
+          const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+          // (Q = 10: after the swap, s / 4 is column bit 9 and the warp-half bit is this lane's l4)
+          const long long j0 = LANE_BIT ? s_hw * 2 * ET + l4 * ET + s_local * 64 + 32 * hw + 2 * W * it
+                                        : s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            const long long j = j0 + 2 * w;
+            float2 gg;
+            // (the full gain's loads are written out here: through at() the compiler spills in this loop)
+            if constexpr (GainT::SEPARABLE) gg = gain.rows2(gcol, j);
+            else gg = make_float2(__ldg(gcol.p + (j << R)), __ldg(gcol.p + ((j + 1) << R)));
+            if constexpr (MODE == 2) {  // dG term: the transformed X column times this one, at rows j, j + 1
+              float* xp = xws + (b << m) + sp + (j << R);
+              const float2 xh = make_float2(__ldcg(xp), __ldcg(xp + (1ll << R)));
+              const float2 pr = mul2(mul2(xh, v[s][w]), sc);
+              if (active) {
+                __stcg(xp, pr.x);
+                __stcg(xp + (1ll << R), pr.y);
+              }
+            }
+            v[s][w] = mul2(v[s][w], mul2(gg, sc));
+          }
+        }
+        if constexpr (LANE_BIT) {
+#pragma unroll
+          for (int t = 0; t < 4; ++t)
+#pragma unroll
+            for (int w = 0; w < W; ++w) bf2(v[t][w], v[t + 4][w]);
+          lane16_swap(v, l4);
+        }
+#pragma unroll
+        for (int hh = 1; hh < NH; hh <<= 1)
+#pragma unroll
+          for (int s = 0; s < NH; ++s)
+            if ((s & hh) == 0)
+#pragma unroll
+              for (int w = 0; w < W; ++w) bf2(v[s][w], v[s + hh][w]);
+#pragma unroll
+        for (int s = 0; s < NH; ++s) {
+          const int s_local = s & (NH / 2 - 1), s_hw = s / (NH / 2);
+          const uint32_t col = s_hw * ET + s_local * 64 + 32 * hw + 2 * W * it;
+#pragma unroll
+          for (int q = 0; q < 2 * W / 16; ++q) {
+            float t[16];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              t[2 * i] = v[s][8 * q + i].x;
+              t[2 * i + 1] = v[s][8 * q + i].y;
+            }
+            tmem_st16(tlane + col + 16 * q, t);
+          }
+        }
+      }  // MODE != 1
     }
     pair_sync(quarter);
-    // round C
+    // round C (MODE 1 stored its column from round B)
 #pragma unroll 1
-    for (int it = 0; it < ITA; ++it) {
+    for (int it = 0; it < (MODE == 1 ? 0 : ITA); ++it) {
       float2 v[64];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {

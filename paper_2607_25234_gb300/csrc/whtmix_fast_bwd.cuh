@@ -1,4 +1,4 @@
-// whtmix_fast_bwd.cuh -- register/TMEM backward kernel for planes of 2^14 <= N*C <= 2^21 elements,
+// whtmix_fast_bwd.cuh -- register/TMEM backward kernel for planes of 2^14 <= N*C <= 2^23 elements,
 // fp32 and bf16 I/O.
 //
 // The backward of the Section III-B mixer Y = W (G o W X) with W = H_N . H_C / sqrt(NC):
@@ -17,8 +17,10 @@
 // column of 2^Q rows as 2^(Q-1) register pairs (j, j + 2^(Q-1)).  For Q <= 6 the transformed X
 // column stays in registers beside the dY column; for Q = 7 (128 rows) it is parked in the
 // thread's TMEM lane (the two warps w and w+4 that share a lane quarter use columns [0, 128) and
-// [128, 256)) while the dY column is transformed.  Because each thread reduces the same dG
-// positions in every group, dG's summation order is exactly b = 0, 1, ..., B-1.
+// [128, 256)) while the dY column is transformed.  Columns of 256 and 512 rows (Q = 8, 9, rows of
+// 2^14) take the forward's TMEM column pass twice: the X columns' bits forward in place, then the
+// dY columns, whose gain step also turns the X column into the product.  Because each thread
+// reduces the same dG positions in every group, dG's summation order is exactly b = 0, 1, ..., B-1.
 #pragma once
 
 #include "whtmix_fast.cuh"
@@ -143,11 +145,11 @@ __device__ __forceinline__ void dg_reduce(float* dg, const float* wsx, int m, lo
 // followed by wsd (P.gp planes).
 template <int D, int R, int Q>
 __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
-  static_assert((R == 13 && Q >= 1 && Q <= 7) || (R == 14 && Q == 7), "supported row/column split");
+  static_assert((R == 13 && Q >= 1 && Q <= 7) || (R == 14 && Q >= 7 && Q <= 9), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   __shared__ uint32_t tmem_slot;
-  constexpr bool USE_TMEM = Q == 7;
+  constexpr bool USE_TMEM = Q >= 7;
   using RW = Row<R>;
   float* sm = reinterpret_cast<float*>(smem_raw);
   const int worker = threadIdx.x / RW::WORKER, wt = threadIdx.x % RW::WORKER;
@@ -164,8 +166,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
-    // lane quarter of this warp; warps w and w + 4 take TMEM columns [0, 128) and [128, 256)
-    tcol = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16) + 128u * (threadIdx.x >> 7);
+    // lane quarter of this warp; for Q = 7 warps w and w + 4 take TMEM columns [0, 128) and
+    // [128, 256); the column passes of Q = 8, 9 split the lane between the two warps themselves
+    tcol = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16) + (Q == 7 ? 128u * (threadIdx.x >> 7) : 0u);
   }
   // tensor memory is allocated before the wait: the previous kernel's CTA on this SM has left
   pdl_wait();
@@ -204,7 +207,15 @@ __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {
       const long long cols = nb << R;
       const long long cb = ((cols * blockIdx.x / gridDim.x) + 4) & ~7ll;
       const long long ce = blockIdx.x + 1 == gridDim.x ? cols : ((cols * (blockIdx.x + 1) / gridDim.x) + 4) & ~7ll;
-      col_pass_bwd<Q, R>(wsx, wsd, g, P.scale, m, cb, ce, tcol);
+      if constexpr (Q >= 8) {
+        // columns of 256 or 512 rows: the X columns' bits forward (stored in place), then the dY
+        // columns with the products written over the X columns at the gain step
+        const FullGain<R> gain{g};
+        col_pass_tmem<Q, R, FullGain<R>, 1>(wsx, gain, P.scale, m, cb, ce, tcol);
+        col_pass_tmem<Q, R, FullGain<R>, 2>(wsd, gain, P.scale, m, cb, ce, tcol, wsx);
+      } else {
+        col_pass_bwd<Q, R>(wsx, wsd, g, P.scale, m, cb, ce, tcol);
+      }
     }
     if (!gsync()) break;
     // phase 3: wsd -> dX, row bits; then this CTA's dG positions

@@ -85,8 +85,9 @@ cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
 // Row bits of the fast forward for a 2^m-element plane.
 inline int forward_row_bits(int) { return 13; }
 
-// Backward: columns of at most 128 rows (the transformed X column of a 128-row column is parked
-// in TMEM), so rows of 2^13 up to 2^20-element planes and rows of 2^14 for 2^21.
+// Backward: rows of 2^13 up to 2^20-element planes (columns of at most 128 rows, the transformed X
+// column of a 128-row column parked in TMEM) and rows of 2^14 from 2^21 (columns of 128, 256 and
+// 512 rows; the TMEM column pass for 256 and 512).
 template <int D>
 cudaError_t launch_backward(const Params& P, int sms, cudaStream_t stream) {
   switch (P.m) {
@@ -98,6 +99,8 @@ cudaError_t launch_backward(const Params& P, int sms, cudaStream_t stream) {
     case 19: return launch_bwd_one<D, 13, 6>(P, sms, stream);
     case 20: return launch_bwd_one<D, 13, 7>(P, sms, stream);
     case 21: return launch_bwd_one<D, 14, 7>(P, sms, stream);
+    case 22: return launch_bwd_one<D, 14, 8>(P, sms, stream);
+    case 23: return launch_bwd_one<D, 14, 9>(P, sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -103,6 +103,11 @@ def test_train_16x8192x256_bf16_forward_backward():
     run_backward(16, 8192, 256, "bf16")
 
 
+def test_fullimage_1x65536x128_bf16_backward_padded():
+    # the full-image shape's training step: 2^23-element planes, rows >= 64800 zero
+    run_backward(1, 65536, 128, "bf16", n_valid=2 * 135 * 240)
+
+
 # ---- shape sweep: single-tile and three-phase plans, aspect ratios, ragged batches ----
 
 SWEEP = [(1, 1, 1), (3, 1, 1), (5, 1, 8), (7, 8, 1), (3, 2, 2), (9, 4, 16), (2, 16, 4), (33, 32, 8),
@@ -124,9 +129,11 @@ def test_forward_sweep(B, N, C, dtype):
 
 BWD_SWEEP = [(1, 1, 1), (3, 4, 2), (5, 32, 16), (2, 64, 128), (6, 512, 16),
              # every column height of the fast backward, N*C = 2^(13+Q) with Q = 1..7 (rows of 2^13)
-             # and 2^21 (rows of 2^14); odd batches leave a short last plane group
+             # and 2^(14+Q) with Q = 7, 8, 9 (rows of 2^14: 2^21, 2^22, 2^23); odd batches leave a
+             # short last plane group
              (3, 128, 128), (2, 8192, 2), (3, 256, 128), (4, 1024, 64), (5, 2048, 64), (2, 64, 4096),
-             (1, 1 << 17, 4), (3, 1024, 1024), (3, 8192, 256), (1, 2, 1 << 20)]
+             (1, 1 << 17, 4), (3, 1024, 1024), (3, 8192, 256), (1, 2, 1 << 20),
+             (3, 16384, 256), (1, 2048, 2048), (2, 65536, 128), (1, 1 << 16, 64)]
 
 
 @pytest.mark.parametrize("B,N,C", BWD_SWEEP)
@@ -213,12 +220,13 @@ def test_in_place_forward_and_backward():
 
 
 def test_backward_is_deterministic():
-    d = inputs.make_inputs(8, 2048, 64, "bf16", seed=7, with_dy=True)
-    x, g, dy = to_dev(d["x"], "bf16"), to_dev(d["g"], "f32"), to_dev(d["dy"], "bf16")
-    a = whtmix.backward(x, g, dy)
-    b = whtmix.backward(x, g, dy)
-    torch.cuda.synchronize()
-    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+    for (B, N, C) in [(8, 2048, 64), (3, 8192, 512)]:   # 128- and 512-row columns
+        d = inputs.make_inputs(B, N, C, "bf16", seed=7, with_dy=True)
+        x, g, dy = to_dev(d["x"], "bf16"), to_dev(d["g"], "f32"), to_dev(d["dy"], "bf16")
+        a = whtmix.backward(x, g, dy)
+        b = whtmix.backward(x, g, dy)
+        torch.cuda.synchronize()
+        assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
     d = inputs.make_inputs(40, 32, 16, "f32", seed=8, with_dy=True)
     x, g, dy = to_dev(d["x"], "f32"), to_dev(d["g"], "f32"), to_dev(d["dy"], "f32")
     a = whtmix.backward(x, g, dy)
