@@ -2,8 +2,9 @@
 //
 // Every check runs before anything is enqueued; a failing call enqueues and writes nothing.
 // The plain calls take their workspace from a per-(device, stream) cache; the _ex calls use the
-// caller's buffer.  Each call is one kernel launch (cooperative when the plan needs device-wide
-// barriers), plus a stream-ordered allocation the first time a cached workspace grows.
+// caller's buffer.  Each call is one kernel launch for most shapes (five per plane group for planes
+// of more than 2^26 elements), with programmatic stream serialisation, plus a stream-ordered
+// allocation the first time a cached workspace grows.
 #include <cuda_runtime.h>
 
 #include <cstring>
@@ -207,17 +208,16 @@ int occupancy(const void* kernel, size_t smem, int* occ_out) {
   return WHTMIX_OK;
 }
 
+// One launch of a generic-engine kernel: a grid of at most the resident CTAs (so that with
+// device-wide barriers, plans M and the backward, every CTA is resident at once).
 template <class K>
-int launch(K kernel, bool cooperative, int sms, long long max_units, size_t smem, const Params& P, cudaStream_t stream) {
+int launch(K kernel, int sms, long long max_units, size_t smem, const Params& P, cudaStream_t stream) {
   cudaError_t e;
   int occ = 0;
   const int rc = occupancy(reinterpret_cast<const void*>(kernel), smem, &occ);
   if (rc != WHTMIX_OK) return rc;
   long long grid = static_cast<long long>(occ) * sms;
   if (max_units < grid) grid = max_units < 1 ? 1 : max_units;
-  // grid <= resident CTAs: with device-wide barriers (plans M and the backward) every CTA is
-  // resident at once
-  (void)cooperative;
   Params p = P;
   void* args[] = {&p};
   e = launch_pdl(reinterpret_cast<const void*>(kernel), static_cast<unsigned>(grid), THREADS, smem, stream, args);
@@ -314,9 +314,9 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
     }
     if (m <= TILE_BITS) {
       const long long ppt = 1ll << (TILE_BITS - m);
-      return launch(k_forward_s<D>, false, sms, (P.B + ppt - 1) / ppt, tile_bytes, P, stream);
+      return launch(k_forward_s<D>, sms, (P.B + ppt - 1) / ppt, tile_bytes, P, stream);
     }
-    return launch(k_forward_m<D>, true, sms, static_cast<long long>(P.gp) << (m - TILE_BITS), tile_bytes, P, stream);
+    return launch(k_forward_m<D>, sms, static_cast<long long>(P.gp) << (m - TILE_BITS), tile_bytes, P, stream);
   }
   if constexpr (D != DT_I32) {
     if (use_fast_backward(D, m)) {
@@ -329,9 +329,9 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
     long long units = (P.gp + ppt - 1) / ppt;
     const long long lunits = ((1ll << m) + THREADS - 1) / THREADS;
     if (lunits > units) units = lunits;
-    return launch(k_backward_s<D>, true, sms, units, 2 * tile_bytes, P, stream);
+    return launch(k_backward_s<D>, sms, units, 2 * tile_bytes, P, stream);
   }
-  return launch(k_backward_m<D>, true, sms, 2ll * (static_cast<long long>(P.gp) << (m - TILE_BITS)), 3 * tile_bytes, P, stream);
+  return launch(k_backward_m<D>, sms, 2ll * (static_cast<long long>(P.gp) << (m - TILE_BITS)), 3 * tile_bytes, P, stream);
 }
 
 // ---- separable log gains (Section III-B, Eq. 2-3): G[n, c] = exp(g_t[n]) exp(g_c[c]) ----

@@ -780,7 +780,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 }
 
 // ---------------------------------------------------------------------------------------------
-// Forward kernel: persistent cooperative grid (one CTA per SM), plane groups of P.gp planes,
+// Forward kernel: persistent grid (one CTA per SM, all resident), plane groups of P.gp planes,
 // three phases.  R and Q are template parameters so that every register array has a static size.
 template <int D, int R, int Q, bool SEP>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {

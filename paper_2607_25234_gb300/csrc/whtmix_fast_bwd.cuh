@@ -141,7 +141,7 @@ __device__ __forceinline__ void dg_reduce(float* dg, const float* wsx, int m, lo
   }
 }
 
-// Backward kernel: persistent cooperative grid (one CTA per SM).  P.ws holds wsx (P.gp planes)
+// Backward kernel: persistent grid (one CTA per SM, all resident).  P.ws holds wsx (P.gp planes)
 // followed by wsd (P.gp planes).
 template <int D, int R, int Q>
 __global__ void __launch_bounds__(THREADS, 1) k_backward_fast(Params P) {

@@ -401,7 +401,7 @@ __global__ void __launch_bounds__(THREADS) k_forward_s(Params P) {
   pdl_trigger();
 }
 
-// Forward, plan M (cooperative launch: device-wide barriers between phases).
+// Forward, plan M (a grid of resident CTAs: device-wide barriers between phases).
 template <int D>
 __global__ void __launch_bounds__(THREADS) k_forward_m(Params P) {
   using A = typename Tr<D>::A;
