@@ -74,7 +74,8 @@ def kernel_name(w) -> str:
 
 
 def backward_kernel_name(w) -> str:
-    """The kernel one whtmix_backward call launches for this workload (mirrors the C ABI's dispatch)."""
+    """The kernel one whtmix_backward call launches for this workload (mirrors the C ABI's dispatch);
+    for the block, the mixer backward inside whtmix_block_backward."""
     m = (w.N * w.C).bit_length() - 1
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 14 if m >= 21 else 13
@@ -102,6 +103,38 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def input_rotation(w, l2: int):
+    """Buffer sets the timed loop rotates over so that their inputs and outputs exceed 3x the L2
+    size (every step then streams from HBM): (sets, bytes per set)."""
+    es = 2 if w.dtype == "bf16" else 4
+    nv = w.n_valid if w.padded_io else w.N
+    plane_b = w.B * nv * w.C * es
+    g_b = (w.N + w.C) * 4 if w.gains == "separable" else w.N * w.C * 4
+    set_bytes = 2 * plane_b + g_b + ((2 * plane_b + g_b) if w.backward else 0)
+    return max(2, -(-3 * l2 // set_bytes)), set_bytes
+
+
+def workload_config(w, world: int, l2: int) -> dict:
+    """The JSON line's config, the same for both arms: the workload and how its steps defeat L2."""
+    nsets, set_bytes = input_rotation(w, l2)
+    return {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype,
+            "gain_dtype": "f32" if w.dtype != "i32" else "i32", "gains": w.gains,
+            "stored_tokens": w.n_valid if w.padded_io else w.N, "parallelism": f"replicas{world}",
+            "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / 2**20:.0f} MiB, "
+                  f"{nsets * set_bytes / l2:.1f}x L2)"}
+
+
+def device_l2_bytes() -> int:
+    """L2 size of GPU 0 (the fallback where none is visible)."""
+    try:
+        import torch
+        if torch.cuda.is_available():
+            return int(getattr(torch.cuda.get_device_properties(0), "L2_cache_size", 0) or 132 * 2**20)
+    except Exception:
+        pass
+    return 132 * 2**20
 
 
 def dist_env():
@@ -233,7 +266,10 @@ def oracle_time_plane(w: inputs.Workload, n_tokens: int, reps: int, threads: int
         else:
             oracle.forward(x, g)
         if dy is not None:
-            oracle.backward(x, g, dy)
+            if w.block:
+                oracle.block_backward(x, w_in, g, w_out, dy)
+            else:
+                oracle.backward(x, g, dy)
         times.append(time.perf_counter() - t)
     oracle.set_threads(1)
     return statistics.median(times), times
@@ -254,17 +290,28 @@ def reference_arm(args, w):
     n = w.N
     while n > 64 and (args.steps + args.warmup) * t_full * n / w.N > budget:
         n //= 2
-    d = inputs.make_inputs(1, n, w.C, w.dtype, seed=0, n_valid=None if w.n_valid is None else min(w.n_valid, n))
+    d = inputs.make_inputs(1, n, w.C, w.dtype, seed=0, n_valid=None if w.n_valid is None else min(w.n_valid, n),
+                           with_dy=w.backward)
     x = inputs.as_float64(d["x"], w.dtype)
     g = d["g"].astype(np.float64)
+    dy = inputs.as_float64(d["dy"], w.dtype) if w.backward else None
     if w.block:
         w_in, w_out = (inputs.as_float64(a, "bf16") for a in inputs.make_projections(w.C, 0))
-        run = lambda: oracle.block_forward(x, w_in, g, w_out)
+        fwd_run = lambda: oracle.block_forward(x, w_in, g, w_out)
+        bwd_run = lambda: oracle.block_backward(x, w_in, g, w_out, dy)
     elif w.gains == "separable":
         g_t, g_c = (a.astype(np.float64) for a in inputs.make_log_gains(n, w.C, 0))
-        run = lambda: oracle.forward_separable(x, g_t, g_c)
+        fwd_run = lambda: oracle.forward_separable(x, g_t, g_c)
+        bwd_run = lambda: oracle.backward_separable(x, g_t, g_c, dy)
     else:
-        run = lambda: oracle.forward(x, g)
+        fwd_run = lambda: oracle.forward(x, g)
+        bwd_run = lambda: oracle.backward(x, g, dy)
+
+    def run():
+        fwd_run()
+        if w.backward:
+            bwd_run()
+
     threads = oracle.set_threads(cores)
     for _ in range(args.warmup):
         run()
@@ -275,13 +322,14 @@ def reference_arm(args, w):
     oracle.set_threads(1)
     value = args.steps * n / el
     sample = (f"per step one [{n},{w.C}] plane of the workload (full plane [{w.N},{w.C}] is {t_full:.2f} s), "
-              f"float64 oracle on {threads} OpenMP threads, CPU {model}")
-    metric = "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
+              f"float64 oracle{' forward + backward' if w.backward else ''} on {threads} OpenMP threads, CPU {model}")
+    metric = ("WHTMix block fwd+bwd tokens/s" if w.backward and w.block else "WHTMix fwd+bwd tokens/s" if w.backward
+              else "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s")
     line = {"impl": "reference", "metric": metric, "value": value, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * el / max(args.steps, 1), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype},
+            "config": workload_config(w, world, device_l2_bytes()),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": sample,
                              "cpu_model": model},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -363,10 +411,7 @@ def ours(args, w):
         dy_host = torch.from_numpy(d["dy"].view(np.int16) if w.dtype == "bf16" else d["dy"])
         if w.dtype == "bf16":
             dy_host = dy_host.view(torch.bfloat16)
-    plane_b = x0.numel() * x0.element_size()
-    g_b = g0.numel() * g0.element_size()
-    set_bytes = 2 * plane_b + g_b + ((2 * plane_b + g_b) if w.backward else 0)
-    nsets = max(2, -(-3 * l2 // set_bytes))
+    nsets, set_bytes = input_rotation(w, l2)
     xs = [x0] + [x0.clone() for _ in range(nsets - 1)]
     gs = [g0] + [g0.clone() for _ in range(nsets - 1)]
     ys = [torch.empty_like(x0) for _ in range(nsets)]
@@ -384,10 +429,18 @@ def ours(args, w):
     fwd_sep = lib.whtmix_forward_separable
     fwd_pad = lib.whtmix_forward_padded
     fwd_block = lib.whtmix_block_forward
-    launches_per_step = 2 if w.backward else 3 if w.block and not block_fused(w) else 1
+    bwd_block = lib.whtmix_block_backward
+    # launches of our kernels per step; the block backward: projection, mixer forward, weight
+    # transpose, projection, two operand transposes, weight gradient and its reduction, mixer
+    # backward, two transposes, weight gradient and reduction, weight transpose, projection
+    block_bwd_launches = 15
+    launches_per_step = ((1 if block_fused(w) else 3) + block_bwd_launches if w.block and w.backward else
+                         2 if w.backward else 3 if w.block and not block_fused(w) else 1)
     if w.block:
         wi = torch.from_numpy(d["w_in"].view(np.int16)).to(dev).view(torch.bfloat16)
         wo = torch.from_numpy(d["w_out"].view(np.int16)).to(dev).view(torch.bfloat16)
+        dwis = [torch.empty(w.C, w.C, dtype=torch.float32, device=dev) for _ in range(nsets)]
+        dwos = [torch.empty(w.C, w.C, dtype=torch.float32, device=dev) for _ in range(nsets)]
 
     def step(i):
         a = args_c[i % nsets]
@@ -403,9 +456,14 @@ def ours(args, w):
             raise whtmix.WhtmixError(rc, "whtmix_forward")
         if w.backward:
             bb = bargs_c[i % nsets]
-            rc = bwd(a[0], a[1], bb[0], bb[1], bb[2], w.B, w.N, w.C, code, sp)
+            if w.block:
+                k = i % nsets
+                rc = bwd_block(a[0], wi.data_ptr(), a[1], wo.data_ptr(), bb[0], bb[1], dwis[k].data_ptr(), bb[2],
+                               dwos[k].data_ptr(), w.B, w.N, w.C, code, sp)
+            else:
+                rc = bwd(a[0], a[1], bb[0], bb[1], bb[2], w.B, w.N, w.C, code, sp)
             if rc != 0:
-                raise whtmix.WhtmixError(rc, "whtmix_backward")
+                raise whtmix.WhtmixError(rc, "whtmix_block_backward" if w.block else "whtmix_backward")
 
     # warm-up (also allocates the cached workspace on this stream)
     for i in range(max(args.warmup, 3)):
@@ -475,6 +533,8 @@ def ours(args, w):
         dyh = dy_host.pin_memory() if w.backward else None
         dxh = torch.empty_like(dyh).pin_memory() if w.backward else None
         dgh = torch.empty_like(gh).pin_memory() if w.backward else None
+        dwih = torch.empty(w.C, w.C).pin_memory() if w.backward and w.block else None
+        dwoh = torch.empty(w.C, w.C).pin_memory() if w.backward and w.block else None
         NB = 2
         s_in, s_comp, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         ev_in = [torch.cuda.Event() for _ in range(NB)]
@@ -491,6 +551,8 @@ def ours(args, w):
             pairs = [(yh, ys[k])]
             if w.backward:
                 pairs += [(dxh, dxs[k]), (dgh, dgs[k])]
+            if w.backward and w.block:
+                pairs += [(dwih, dwis[k]), (dwoh, dwos[k])]
             return pairs
 
         def e2e_step(i):
@@ -514,7 +576,9 @@ def ours(args, w):
                     whtmix.forward_padded(xd, gd, out=yd)
                 else:
                     whtmix.forward(xd, gd, out=yd)
-                if w.backward:
+                if w.backward and w.block:
+                    whtmix.block_backward(xd, wi, gd, wo, dys[k], dx=dxs[k], dw_in=dwis[k], dg=dgs[k], dw_out=dwos[k])
+                elif w.backward:
                     whtmix.backward(xd, gd, dys[k], dx=dxs[k], dg=dgs[k])
                 ev_comp[k].record(s_comp)
             with torch.cuda.stream(s_out):
@@ -565,16 +629,13 @@ def ours(args, w):
                                  "sample": f"the same plane on one thread, median of {len(times_one)} run(s): "
                                            + ", ".join(f"{t:.3f}" for t in times_one) + " s"}}
 
-    metric = "WHTMix fwd+bwd tokens/s" if w.backward else "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s"
+    metric = ("WHTMix block fwd+bwd tokens/s" if w.backward and w.block else "WHTMix fwd+bwd tokens/s" if w.backward
+              else "WHTMix block fwd tokens/s" if w.block else "WHTMix fwd tokens/s")
     line = {"metric": metric, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "i32" if w.dtype == "i32" else "f32",
             "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "N": w.N, "C": w.C, "io_dtype": w.dtype, "gain_dtype":
-                       "f32" if w.dtype != "i32" else "i32", "gains": w.gains, "stored_tokens": nv,
-                       "parallelism": f"replicas{world}",
-                       "l2": f"inputs rotate over {nsets} buffer sets ({nsets * set_bytes / 2**20:.0f} MiB, "
-                             f"{nsets * set_bytes / l2:.1f}x L2)"},
+            "config": workload_config(w, world, l2),
             "hbm_gbs": achieved, "pct_of_measured_peak": 100.0 * achieved / peak,
             "pct_of_nominal_peak": 100.0 * achieved / NOMINAL_HBM_GBS,
             "kernel_us": {"per_step": 1e3 * step_ms,

@@ -146,6 +146,10 @@ WORKLOADS = {
     "fullimage_train_1x65536x128_bf16": Workload("fullimage_train_1x65536x128_bf16", 1, 65536, 128, "bf16",
                                                  backward=True, n_valid=2 * 135 * 240,
                                                  description="full-image shape, training step: forward + backward"),
+    # the whole block's training step: block forward + block backward (weight gradients included)
+    "block_train_fullimage_1x65536x128_bf16": Workload("block_train_fullimage_1x65536x128_bf16", 1, 65536, 128, "bf16",
+                                                       backward=True, n_valid=2 * 135 * 240, block=True,
+                                                       description="mixer block, training step: forward + backward"),
     # the paper's mixer as trained: separable log gains and in-library padding
     "fullimage_paper_1x64800x128_bf16": Workload("fullimage_paper_1x64800x128_bf16", 1, 65536, 128, "bf16",
                                                  n_valid=2 * 135 * 240, padded_io=True, gains="separable",

@@ -95,3 +95,24 @@ def test_clock_summary_uses_the_timed_window_and_decodes_reasons():
     assert s.summary(10.0, 11.0)["window"] == "whole_run"   # nothing inside: every sample, marked so
     empty = bench.ClockSampler("0").summary(0.0, 1.0)
     assert empty["samples"] == 0 and empty["sm_mhz"] is None
+
+
+def test_reference_arm_line_matches_ours_in_config_and_metric(monkeypatch, capsys):
+    """The driver compares the two arms' lines: the reference arm (the CPU oracle) reports the same
+    config (built by the same function as the GPU arm's) and, for a training step, the same
+    forward + backward metric."""
+    for k in ("WORLD_SIZE", "RANK", "LOCAL_RANK"):
+        monkeypatch.delenv(k, raising=False)
+
+    class Args:
+        steps, warmup, gpus = 1, 1, 1
+    for name, metric in (("tiny_1x256x64_f32", "WHTMix fwd tokens/s"),
+                         ("train_16x8192x256_bf16", "WHTMix fwd+bwd tokens/s")):
+        w = W[name]
+        small = w if w.B * w.N * w.C <= 1 << 16 else \
+            bench.inputs.Workload(w.name, 1, 256, w.C, w.dtype, backward=w.backward)
+        bench.reference_arm(Args(), small)
+        line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+        assert line["impl"] == "reference" and line["metric"] == metric
+        assert line["config"] == bench.workload_config(small, 1, bench.device_l2_bytes())
+        assert line["cpu_baseline"]["cores"] >= 1 and line["value"] > 0
