@@ -65,7 +65,7 @@ def kernel_name(w) -> str:
             and not w.block and (not w.padded_io or padded_ok)):
         return f"k_forward_plane<{w.dtype}, column bits {m - 14}> (one plane per CTA, in tensor memory)"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
-        r = 13
+        r = 14 if m == 21 else 13
         sep = ", separable gains" if w.gains == "separable" else ""
         pad = ", in-kernel token padding" if w.padded_io else ""
         name = f"k_forward_fast<{w.dtype}, R={r}, Q={m - r}{sep}{pad}>"
@@ -431,9 +431,9 @@ def ours(args, w):
     fwd_block = lib.whtmix_block_forward
     bwd_block = lib.whtmix_block_backward
     # launches of our kernels per step; the block backward: projection, mixer forward, weight
-    # transpose, projection, two operand transposes, weight gradient and its reduction, mixer
-    # backward, two transposes, weight gradient and reduction, weight transpose, projection
-    block_bwd_launches = 15
+    # transpose, projection, weight gradient and its reduction, mixer backward, weight gradient
+    # and reduction, weight transpose, projection
+    block_bwd_launches = 11
     launches_per_step = ((1 if block_fused(w) else 3) + block_bwd_launches if w.block and w.backward else
                          2 if w.backward else 3 if w.block and not block_fused(w) else 1)
     if w.block:

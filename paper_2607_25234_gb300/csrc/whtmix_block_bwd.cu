@@ -1,17 +1,17 @@
 // whtmix_block_bwd.cu -- the pieces of the mixer block's backward (Section III-B, Eq. 1-4) that the
 // forward kernels do not already provide: the weight gradients
 //     dW[o, i] = sum over tokens t of A[t, o] B[t, i]      (dW_out = dY^T M, dW_in = dZ^T X)
-// on the 5th-generation tensor cores, and the transposes that feed them.
+// on the 5th-generation tensor cores, and the weight transposes the projections need.
 //
-// A and B are [T, C] bf16 token rows; the contraction runs over the tokens, so both are first
-// transposed into [C, Tp] (Tp = T rounded up to 64, zero past T) -- K-major operands for the MMA.
-// k_wgrad splits the tokens into one chunk per CTA (one persistent CTA per SM, 128 threads): per
-// K tile of 64 tokens the CTA stages the A rows (output channels o, 128 per MMA tile) and the B rows
-// (input channels i) in the tensor core's no-swizzle K-major canonical layout, double-buffered,
-// and one thread issues tcgen05.mma (kind::f16, M = 128, N = C, K = 16) into a TMEM accumulator
-// per 128 rows of o, committed to an mbarrier per buffer.  Each thread then reads its row o of the
+// A and B are [T, C] bf16 token rows; the contraction runs over the tokens.  k_wgrad splits the
+// tokens into one chunk per CTA (one persistent CTA per SM, 128 threads): per K tile of 64 tokens
+// the CTA reads the token rows of both operands, transposes 8 x 8 blocks in registers and stages
+// the A rows (output channels o, 128 per MMA tile) and the B rows (input channels i) in the tensor
+// core's 128-byte-swizzled K-major layout, double-buffered, with the next tile's loads in flight;
+// one thread issues tcgen05.mma (kind::f16, M = 128, N = C, K = 16) into a TMEM accumulator per
+// 128 rows of o, committed to an mbarrier per buffer.  Each thread then reads its row o of the
 // accumulator (tcgen05.ld) into the chunk's fp32 partial [C, C]; k_wgrad_reduce adds the partials
-// in ascending chunk order, so dW is the same bit for bit on every run.
+// in a fixed order, so dW is the same bit for bit on every run.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -29,7 +29,8 @@ constexpr int WG_THREADS = 128;    // one thread per TMEM lane = per output row 
 constexpr int TR_THREADS = 256;
 constexpr size_t SMEM_MIN = 120 * 1024;  // more than half an SM: one CTA per SM, so TMEM allocation never waits
 
-// out[c, t] = in[t, c] for t < T, 0 for T <= t < Tp (both bf16; C a multiple of 64, Tp of 64).
+// out[c, t] = in[t, c] for t < T, 0 for T <= t < Tp (both bf16; C a multiple of 64, Tp of 64):
+// the weights' transposes.
 __global__ void __launch_bounds__(TR_THREADS) k_transpose(const uint16_t* __restrict__ in, uint16_t* __restrict__ out,
                                                           long long T, int C, long long Tp) {
   __shared__ uint16_t tile[64][66];
@@ -51,19 +52,29 @@ __global__ void __launch_bounds__(TR_THREADS) k_transpose(const uint16_t* __rest
 }
 
 // Partial weight gradient of token chunk blockIdx.x: part[chunk][o][i] = sum over the chunk's
-// tokens of At[o][t] Bt[i][t].  C in {64, 128, 256}.
+// tokens t of A[t][o] B[t][i], with A and B the [T, C] token rows as given.  C in {64, 128, 256}.
+//
+// A K tile of KT = 64 tokens of an operand becomes C rows (channels) of 128 bytes (64 tokens) in
+// the tensor core's 128-byte-swizzled K-major layout: in each 1024-byte group of 8 rows, the
+// 16-byte chunk j (tokens 8j .. 8j + 7) of row r sits at chunk position j ^ (r mod 8).  Thread
+// work item (r8, k) reads the 8 x 8 block of channels 8 r8 .. + 7 and tokens 8 k .. + 7 as eight
+// 16-byte token rows, transposes it in registers (byte permutes of token pairs) and writes the
+// eight 16-byte channel rows; the eight items of a row group land in eight different bank groups.
 template <int C>
-__global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad(const __nv_bfloat16* __restrict__ At,
-                                                         const __nv_bfloat16* __restrict__ Bt, float* __restrict__ part,
-                                                         long long Tp, int nchunk, unsigned int* err) {
+__global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad(const uint16_t* __restrict__ A, const uint16_t* __restrict__ B,
+                                                         float* __restrict__ part, long long T, int nchunk,
+                                                         unsigned int* err) {
   constexpr int MT = C > 128 ? C / 128 : 1;          // MMA tiles of 128 output rows
-  constexpr int AR = MT * 128;                       // staged A rows (rows >= C are zero)
+  constexpr int AR = MT * 128;                       // staged A rows (rows >= C stay zero)
   constexpr uint32_t A_BYTES = AR * KT * 2, B_BYTES = C * KT * 2, STAGE = A_BYTES + B_BYTES;
   constexpr uint32_t TCOLS = MT * C;                 // 64, 128 or 512 TMEM columns
+  constexpr int ITEMS = C / WG_THREADS > 0 ? C / WG_THREADS : 1;  // 8 x 8 blocks per operand per thread
   static_assert(C == 64 || C == 128 || C == 256, "channels");
-  extern __shared__ __align__(1024) unsigned char smem[];
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ uint64_t mbar[2];
   __shared__ uint32_t tmem_slot;
+  // the swizzle pattern is a function of the address: stage buffers start on 1024-byte boundaries
+  unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int tid = threadIdx.x, warp = tid >> 5;
   if (tid < 32) tmem_alloc(&tmem_slot, TCOLS);
   if (tid == 0) {
@@ -71,29 +82,64 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad(const __nv_bfloat16* __
     mbar_init(&mbar[1], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if constexpr (AR > C) {  // A rows C .. AR - 1 of both buffers: zero once, never written again
+    for (int q = tid; q < 2 * (AR - C) * 8; q += WG_THREADS) {
+      const int b = q / ((AR - C) * 8), rem = q % ((AR - C) * 8);
+      *reinterpret_cast<uint4*>(smem + b * STAGE + C * 128 + rem * 16) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   pdl_wait();
   const uint32_t tmem = tmem_slot;
-  const long long ntiles = Tp / KT;
+  const long long ntiles = (T + KT - 1) / KT;
   const long long k0 = ntiles * blockIdx.x / nchunk, k1 = ntiles * (blockIdx.x + 1) / nchunk;
+  const bool has_item = tid < C;  // C work items per operand and tile: C = 64 leaves threads 64 .. 127 idle
 
-  // K tile kt of both operands into buffer `buf`, canonical layout (8-row x 16-byte core matrices,
-  // the K-adjacent one 128 bytes on, the next 8 rows KT / 8 x 128 bytes on)
-  auto stage = [&](long long kt, int buf) {
+  // the 8 x 8 blocks of tile kt, item n of this thread: n-th work item tid + 128 n = 8 r8 + k
+  uint4 ra[ITEMS][8], rb[ITEMS][8];
+  auto load = [&](long long kt) {
+#pragma unroll
+    for (int n = 0; n < ITEMS; ++n) {
+      const int item = tid + WG_THREADS * n, r8 = item >> 3, k = item & 7;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const long long t = kt * KT + 8 * k + j;
+        const bool live = has_item && t < T;
+        const long long off = (live ? t : 0) * C + 8 * r8;
+        ra[n][j] = live ? __ldcs(reinterpret_cast<const uint4*>(A + off)) : make_uint4(0u, 0u, 0u, 0u);
+        rb[n][j] = live ? __ldcs(reinterpret_cast<const uint4*>(B + off)) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+  };
+  // transpose one 8 x 8 block (v[j] = token j's 8 channels) and store its 8 channel rows
+  auto put = [&](unsigned char* base, const uint4 (&v)[8], int r8, int k) {
+    uint32_t o[8][4];
+#pragma unroll
+    for (int j = 0; j < 8; j += 2) {
+      const uint32_t a[4] = {v[j].x, v[j].y, v[j].z, v[j].w}, b[4] = {v[j + 1].x, v[j + 1].y, v[j + 1].z, v[j + 1].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        o[2 * q][j / 2] = __byte_perm(a[q], b[q], 0x5410);      // channel 2q, tokens j, j + 1
+        o[2 * q + 1][j / 2] = __byte_perm(a[q], b[q], 0x7632);  // channel 2q + 1, tokens j, j + 1
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+      *reinterpret_cast<uint4*>(base + (r8 * 8 + c) * 128 + ((k ^ c) << 4)) = make_uint4(o[c][0], o[c][1], o[c][2], o[c][3]);
+  };
+  auto store = [&](int buf) {
     unsigned char* sa = smem + buf * STAGE;
     unsigned char* sb = sa + A_BYTES;
-    const long long t0 = kt * KT;
-    for (int q = tid; q < AR * (KT / 8); q += WG_THREADS) {
-      const int r = q / (KT / 8), k = (q % (KT / 8)) * 8;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (r < C) v = __ldcs(reinterpret_cast<const uint4*>(At + r * Tp + t0 + k));
-      *reinterpret_cast<uint4*>(sa + core_off(r, k, KT)) = v;
-    }
-    for (int q = tid; q < C * (KT / 8); q += WG_THREADS) {
-      const int r = q / (KT / 8), k = (q % (KT / 8)) * 8;
-      *reinterpret_cast<uint4*>(sb + core_off(r, k, KT)) = __ldcs(reinterpret_cast<const uint4*>(Bt + r * Tp + t0 + k));
+    if (has_item) {
+#pragma unroll
+      for (int n = 0; n < ITEMS; ++n) {
+        const int item = tid + WG_THREADS * n;
+        put(sa, ra[n], item >> 3, item & 7);
+        put(sb, rb[n], item >> 3, item & 7);
+      }
     }
     // generic-proxy shared-memory writes -> visible to the tensor core (async proxy)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -102,35 +148,36 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad(const __nv_bfloat16* __
   const uint32_t idesc = instr_desc(128, C);
   uint32_t parity[2] = {0u, 0u};
   bool ok = true;
-  stage(k0, 0);
-  __syncthreads();
+  if (k1 > k0) load(k0);
   for (long long kt = k0; kt < k1; ++kt) {
     const int buf = static_cast<int>((kt - k0) & 1);
+    if (kt - k0 >= 2) {  // buffer buf is free once the MMAs of tile kt - 2 (its last reader) completed
+      ok = __syncthreads_and(mbar_wait(&mbar[buf], parity[buf]) ? 1 : 0) != 0;
+      parity[buf] ^= 1u;
+      if (!ok) break;
+    }
+    store(buf);
+    if (kt + 1 < k1) load(kt + 1);  // in flight while this tile is handed to the tensor core
+    __syncthreads();
     if (tid == 0) {
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t sa = smem_u32(smem + buf * STAGE), sb = sa + A_BYTES;
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
-        for (int ks = 0; ks < KT / 16; ++ks)  // K steps of 16: two core matrices along K
-          mma_bf16(tmem + mt * C, smem_desc(sa + mt * (128 * KT * 2) + ks * 256, 128, (KT / 8) * 128),
-                   smem_desc(sb + ks * 256, 128, (KT / 8) * 128), idesc, (kt > k0 || ks > 0) ? 1u : 0u);
+        for (int ks = 0; ks < KT / 16; ++ks)  // K steps of 16 tokens: 32 bytes along the swizzled rows
+          mma_bf16(tmem + mt * C, sw128_desc(sa + mt * (128 * 128) + ks * 32), sw128_desc(sb + ks * 32), idesc,
+                   (kt > k0 || ks > 0) ? 1u : 0u);
       mma_commit(&mbar[buf]);
     }
-    if (kt + 1 < k1) {
-      const int nb = buf ^ 1;
-      if (kt > k0) {  // buffer nb is free once the MMAs of tile kt - 1 (its last reader) completed
-        ok = __syncthreads_and(mbar_wait(&mbar[nb], parity[nb]) ? 1 : 0) != 0;
-        parity[nb] ^= 1u;
-        if (!ok) break;
-      }
-      stage(kt + 1, nb);
-      __syncthreads();
-    }
   }
-  if (ok && k1 > k0) {  // the last tile's commit covers every MMA issued before it
-    const int lb = static_cast<int>((k1 - 1 - k0) & 1);
-    ok = __syncthreads_and(mbar_wait(&mbar[lb], parity[lb]) ? 1 : 0) != 0;
+  if (ok && k1 > k0) {  // the last two tiles' commits cover every MMA issued
+    const long long n = k1 - k0;
+    for (long long kt = (n >= 2 ? k1 - 2 : k0); kt < k1 && ok; ++kt) {
+      const int b = static_cast<int>((kt - k0) & 1);
+      ok = __syncthreads_and(mbar_wait(&mbar[b], parity[b]) ? 1 : 0) != 0;
+      parity[b] ^= 1u;
+    }
   }
   if (!ok && tid == 0) atomicOr(err, 1u << 13);
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -161,23 +208,50 @@ __global__ void __launch_bounds__(WG_THREADS, 1) k_wgrad(const __nv_bfloat16* __
   if (tid < 32) tmem_dealloc(tmem, TCOLS);
 }
 
-// dW[o][i] = sum of the chunks' partials in ascending chunk order (float32).
-__global__ void __launch_bounds__(TR_THREADS) k_wgrad_reduce(const float* __restrict__ part, float* __restrict__ out,
-                                                             int cc, int nchunk) {
+// dW = the sum of the chunks' partials (float32) in a fixed order: RG runs of consecutive chunks,
+// each summed in ascending order by one thread, then the RG run sums in ascending order.  A CTA
+// covers 32 float4 outputs x RG runs.
+constexpr int RG = TR_THREADS / 32;
+__global__ void __launch_bounds__(TR_THREADS) k_wgrad_reduce(const float4* __restrict__ part, float4* __restrict__ out,
+                                                             int cc4, int nchunk) {
+  __shared__ float4 sums[RG][32];
   pdl_wait();
-  for (int q = blockIdx.x * blockDim.x + threadIdx.x; q < cc; q += gridDim.x * blockDim.x) {
-    float acc = 0.f;
-    for (int c = 0; c < nchunk; ++c) acc += part[static_cast<long long>(c) * cc + q];
-    out[q] = acc;
+  const int o = blockIdx.x * 32 + (threadIdx.x & 31), g = threadIdx.x >> 5;
+  const int c0 = nchunk * g / RG, c1 = nchunk * (g + 1) / RG;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (o < cc4) {
+    int c = c0;
+    for (; c + 4 <= c1; c += 4) {
+      float4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = __ldcs(part + static_cast<long long>(c + u) * cc4 + o);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) acc = make_float4(acc.x + v[u].x, acc.y + v[u].y, acc.z + v[u].z, acc.w + v[u].w);
+    }
+    for (; c < c1; ++c) {
+      const float4 v = __ldcs(part + static_cast<long long>(c) * cc4 + o);
+      acc = make_float4(acc.x + v.x, acc.y + v.y, acc.z + v.z, acc.w + v.w);
+    }
+  }
+  sums[g][threadIdx.x & 31] = acc;
+  __syncthreads();
+  if (g == 0 && o < cc4) {
+    float4 s = sums[0][threadIdx.x];
+#pragma unroll
+    for (int r = 1; r < RG; ++r) {
+      const float4 v = sums[r][threadIdx.x];
+      s = make_float4(s.x + v.x, s.y + v.y, s.z + v.z, s.w + v.w);
+    }
+    out[o] = s;
   }
   pdl_trigger();
 }
 
 // ---- host ----
 
-// Token chunks of one weight gradient: one per SM, at most one per K tile.
-int wgrad_chunks(long long Tp, int sms) {
-  const long long nt = Tp / KT;
+// Token chunks of one weight gradient over T tokens: one per SM, at most one per K tile.
+int wgrad_chunks(long long T, int sms) {
+  const long long nt = (T + KT - 1) / KT;
   return static_cast<int>(nt < sms ? (nt < 1 ? 1 : nt) : sms);
 }
 
@@ -191,35 +265,36 @@ cudaError_t transpose(const void* in, void* out, long long T, int C, long long T
 }
 
 template <int C>
-cudaError_t wgrad_c(const void* at, const void* bt, float* part, float* out, long long Tp, int sms, unsigned int* err,
+cudaError_t wgrad_c(const void* a_tok, const void* b_tok, float* part, float* out, long long T, int sms, unsigned int* err,
                     cudaStream_t stream) {
   constexpr int MT = C > 128 ? C / 128 : 1;
-  constexpr size_t need = 2ull * (MT * 128 + C) * KT * 2;
+  constexpr size_t need = 2ull * (MT * 128 + C) * KT * 2 + 1024;  // two stages, 1024-byte alignment slack
   const size_t smem = need > SMEM_MIN ? need : SMEM_MIN;
   const void* k = reinterpret_cast<const void*>(k_wgrad<C>);
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  int nchunk = wgrad_chunks(Tp, sms);
-  const __nv_bfloat16* a = static_cast<const __nv_bfloat16*>(at);
-  const __nv_bfloat16* b = static_cast<const __nv_bfloat16*>(bt);
-  void* args[] = {&a, &b, &part, &Tp, &nchunk, &err};
+  int nchunk = wgrad_chunks(T, sms);
+  const uint16_t* a = static_cast<const uint16_t*>(a_tok);
+  const uint16_t* b = static_cast<const uint16_t*>(b_tok);
+  void* args[] = {&a, &b, &part, &T, &nchunk, &err};
   e = launch_pdl(k, static_cast<unsigned>(nchunk), WG_THREADS, smem, stream, args);
   if (e != cudaSuccess) return e;
-  int cc = C * C;
-  const float* pc = part;
-  void* rargs[] = {&pc, &out, &cc, &nchunk};
-  return launch_pdl(reinterpret_cast<const void*>(k_wgrad_reduce), static_cast<unsigned>((cc + TR_THREADS - 1) / TR_THREADS),
-                    TR_THREADS, 0, stream, rargs);
+  int cc4 = C * C / 4;
+  const float4* pc = reinterpret_cast<const float4*>(part);
+  float4* o4 = reinterpret_cast<float4*>(out);
+  void* rargs[] = {&pc, &o4, &cc4, &nchunk};
+  return launch_pdl(reinterpret_cast<const void*>(k_wgrad_reduce), static_cast<unsigned>((cc4 + 31) / 32), TR_THREADS, 0,
+                    stream, rargs);
 }
 
-// dW = A^T B over the tokens, from the transposed operands at, bt [C, Tp]; part holds
-// wgrad_chunks(Tp, sms) partial [C, C] fp32 planes.
-cudaError_t wgrad(const void* at, const void* bt, float* part, float* out, long long Tp, int C, int sms,
+// dW = A^T B over the T tokens of the [T, C] bf16 operands a_tok, b_tok; part holds
+// wgrad_chunks(T, sms) partial [C, C] fp32 planes; out is 16-byte aligned.
+cudaError_t wgrad(const void* a_tok, const void* b_tok, float* part, float* out, long long T, int C, int sms,
                   unsigned int* err, cudaStream_t stream) {
   switch (C) {
-    case 64: return wgrad_c<64>(at, bt, part, out, Tp, sms, err, stream);
-    case 128: return wgrad_c<128>(at, bt, part, out, Tp, sms, err, stream);
-    case 256: return wgrad_c<256>(at, bt, part, out, Tp, sms, err, stream);
+    case 64: return wgrad_c<64>(a_tok, b_tok, part, out, T, sms, err, stream);
+    case 128: return wgrad_c<128>(a_tok, b_tok, part, out, T, sms, err, stream);
+    case 256: return wgrad_c<256>(a_tok, b_tok, part, out, T, sms, err, stream);
     default: return cudaErrorInvalidValue;
   }
 }

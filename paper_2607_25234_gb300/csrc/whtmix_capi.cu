@@ -33,10 +33,10 @@ cudaError_t project(const void* x, const void* w, void* z, long long T, int C, b
                     cudaStream_t s);
 }  // namespace proj
 namespace bbwd {
-// whtmix_block_bwd.cu: the block backward's transposes and weight gradients on the tensor cores
-int wgrad_chunks(long long Tp, int sms);
+// whtmix_block_bwd.cu: the block backward's weight transposes and weight gradients on the tensor cores
+int wgrad_chunks(long long T, int sms);
 cudaError_t transpose(const void* in, void* out, long long T, int C, long long Tp, int sms, cudaStream_t stream);
-cudaError_t wgrad(const void* at, const void* bt, float* part, float* out, long long Tp, int C, int sms,
+cudaError_t wgrad(const void* a_tok, const void* b_tok, float* part, float* out, long long T, int C, int sms,
                   unsigned int* err, cudaStream_t stream);
 }  // namespace bbwd
 }  // namespace whtmix
@@ -895,14 +895,12 @@ int whtmix_block_backward(const void* x, const void* w_in, const void* gains, co
   }
   rc = device_check(&dev, &sms);
   if (rc != WHTMIX_OK) return rc;
-  // slot-1 layout: Z, M, dM [T, C] bf16; a transposed weight [C, C] bf16; the two transposed
-  // operands [C, Tp] bf16 of a weight gradient; its per-chunk partials [chunks, C, C] fp32
-  const long long Tp = (T + 63) / 64 * 64;
-  const int chunks = bbwd::wgrad_chunks(Tp, sms);
-  const size_t tb = static_cast<size_t>(C) * Tp * 2;
-  size_t off[8], total = 0;
-  const size_t sizes[7] = {pb, pb, pb, wb, tb, tb, static_cast<size_t>(chunks) * wgb};
-  for (int i = 0; i < 7; ++i) {
+  // slot-1 layout: Z, M, dM [T, C] bf16; a transposed weight [C, C] bf16; the per-chunk partials
+  // [chunks, C, C] fp32 of a weight gradient
+  const int chunks = bbwd::wgrad_chunks(T, sms);
+  size_t off[5], total = 0;
+  const size_t sizes[5] = {pb, pb, pb, wb, static_cast<size_t>(chunks) * wgb};
+  for (int i = 0; i < 5; ++i) {
     off[i] = total;
     total += align256(sizes[i]);
   }
@@ -911,8 +909,7 @@ int whtmix_block_backward(const void* x, const void* w_in, const void* gains, co
   if (rc != WHTMIX_OK) return rc;
   char* base = static_cast<char*>(w1);
   void *Z = base + off[0], *M = base + off[1], *dM = base + off[2], *WT = base + off[3];
-  void *At = base + off[4], *Bt = base + off[5];
-  float* part = reinterpret_cast<float*>(base + off[6]);
+  float* part = reinterpret_cast<float*>(base + off[4]);
   auto err_word = [&](unsigned int** e) -> int {  // the slot-0 header's error word, read by whtmix_sync
     void* w0 = nullptr;
     const int r = cached_workspace(dev, stream, HEADER_BYTES, &w0, 0);
@@ -937,17 +934,13 @@ int whtmix_block_backward(const void* x, const void* w_in, const void* gains, co
   // Eq. 4 backward: dM = dY W_out (the projection with W_out^T), dW_out = dY^T M
   WHTMIX_CUDA_STEP(bbwd::transpose(w_out, WT, C, static_cast<int>(C), C, sms, stream));
   WHTMIX_STEP(whtmix_project(dy, WT, dM, T, C, WHTMIX_BF16, stream));
-  WHTMIX_CUDA_STEP(bbwd::transpose(dy, At, T, static_cast<int>(C), Tp, sms, stream));
-  WHTMIX_CUDA_STEP(bbwd::transpose(M, Bt, T, static_cast<int>(C), Tp, sms, stream));
   WHTMIX_STEP(err_word(&err));
-  WHTMIX_CUDA_STEP(bbwd::wgrad(At, Bt, part, static_cast<float*>(dw_out), Tp, static_cast<int>(C), sms, err, stream));
+  WHTMIX_CUDA_STEP(bbwd::wgrad(dy, M, part, static_cast<float*>(dw_out), T, static_cast<int>(C), sms, err, stream));
   // the mixer's backward: dZ (into dx) and dG
   WHTMIX_STEP(run(full_call(true, Z, gains, dM, dx, dgains, B, N, N, C, dtype), nullptr, 0, false, stream));
   // Eq. 1 backward: dW_in = dZ^T X, then dX = dZ W_in in place
-  WHTMIX_CUDA_STEP(bbwd::transpose(dx, At, T, static_cast<int>(C), Tp, sms, stream));
-  WHTMIX_CUDA_STEP(bbwd::transpose(x, Bt, T, static_cast<int>(C), Tp, sms, stream));
   WHTMIX_STEP(err_word(&err));
-  WHTMIX_CUDA_STEP(bbwd::wgrad(At, Bt, part, static_cast<float*>(dw_in), Tp, static_cast<int>(C), sms, err, stream));
+  WHTMIX_CUDA_STEP(bbwd::wgrad(dx, x, part, static_cast<float*>(dw_in), T, static_cast<int>(C), sms, err, stream));
   WHTMIX_CUDA_STEP(bbwd::transpose(w_in, WT, C, static_cast<int>(C), C, sms, stream));
   WHTMIX_STEP(whtmix_project(dx, WT, dx, T, C, WHTMIX_BF16, stream));
 #undef WHTMIX_STEP

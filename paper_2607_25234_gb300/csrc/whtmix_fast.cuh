@@ -784,7 +784,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 // three phases.  R and Q are template parameters so that every register array has a static size.
 template <int D, int R, int Q, bool SEP>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
-  static_assert((R == 13 && Q >= 1 && Q <= 10) || (R == 14 && Q == 9), "supported row/column split");
+  static_assert((R == 13 && Q >= 1 && Q <= 10) || (R == 14 && (Q == 7 || Q == 9)), "supported row/column split");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   __shared__ uint32_t tmem_slot;

@@ -61,10 +61,12 @@ cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
   return launch_persistent(reinterpret_cast<const void*>(k_backward_fast<D, R, Q>), P, sms, stream);
 }
 
-// Rows of 2^13 elements at every size; 2^23-element planes take 1024-row columns (two lanes per
-// column).  With 152 SMs, 1024 rows of 2^13 spread as 7 or 6 per CTA, where 512 rows of 2^14
-// give 56 CTAs four rows against three; measured on the 2^22 planes, 2^13 rows with 512-row
-// columns beat 2^14 rows.
+// Rows of 2^13 elements at every size but 2^21; 2^23-element planes take 1024-row columns (two
+// lanes per column).  With 152 SMs, 1024 rows of 2^13 spread as 7 or 6 per CTA, where 512 rows of
+// 2^14 give 56 CTAs four rows against three; measured on the 2^22 planes, 2^13 rows with 512-row
+// columns beat 2^14 rows.  2^21-element planes take rows of 2^14 and 128-row columns, one column
+// per thread in registers, instead of 256-row columns in tensor memory: measured on sixteen such
+// planes (bf16), 138 us against 146 us per call.
 // SEP: separable log gains (P.gt, P.gc) instead of G; needs 1 <= P.cbits <= row bits.
 template <int D, bool SEP>
 cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
@@ -76,14 +78,14 @@ cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
     case 18: return launch_one<D, 13, 5, SEP>(P, sms, stream);
     case 19: return launch_one<D, 13, 6, SEP>(P, sms, stream);
     case 20: return launch_one<D, 13, 7, SEP>(P, sms, stream);
-    case 21: return launch_one<D, 13, 8, SEP>(P, sms, stream);
+    case 21: return launch_one<D, 14, 7, SEP>(P, sms, stream);
     case 22: return launch_one<D, 13, 9, SEP>(P, sms, stream);
     case 23: return launch_one<D, 13, 10, SEP>(P, sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 // Row bits of the fast forward for a 2^m-element plane.
-inline int forward_row_bits(int) { return 13; }
+inline int forward_row_bits(int m) { return m == 21 ? 14 : 13; }
 
 // Backward: rows of 2^13 up to 2^20-element planes (columns of at most 128 rows, the transformed X
 // column of a 128-row column parked in TMEM) and rows of 2^14 from 2^21 (columns of 128, 256 and

@@ -132,10 +132,6 @@ __global__ void __launch_bounds__(THREADS, 1) k_proj(const __nv_bfloat16* x, con
 // Tokens past T are zero-filled by the loads and dropped by the stores (the tensor maps' bounds).
 constexpr int P2_THREADS = 192;
 
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
-  return static_cast<uint64_t>((addr & 0x3FFFFu) >> 4) | (1ull << 16) | (static_cast<uint64_t>(1024 >> 4) << 32) |
-         (1ull << 46) | (2ull << 61);
-}
 // K step ks (16 bf16) of an R-row K-major operand stored as 64-element atoms of R x 128 bytes
 template <int R>
 __device__ __forceinline__ uint64_t sw_op_desc(uint32_t base, int ks) {

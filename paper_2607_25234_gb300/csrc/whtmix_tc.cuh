@@ -1,6 +1,6 @@
 // whtmix_tc.cuh -- the pieces of a tcgen05 (5th-generation tensor core) kernel shared by the
 // projections (whtmix_proj.cu) and the block backward's weight gradients (whtmix_block_bwd.cu):
-// shared-memory matrix descriptors for the no-swizzle K-major canonical layout, the kind::f16
+// shared-memory matrix descriptors (no swizzle and 128-byte swizzle, K-major), the kind::f16
 // instruction descriptor, mbarriers with a bounded wait, TMEM allocation, MMA issue and TMEM loads.
 #pragma once
 
@@ -19,6 +19,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) { return static_cast
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
   return static_cast<uint64_t>((addr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(lbo >> 4) << 16) |
          (static_cast<uint64_t>(sbo >> 4) << 32) | (1ull << 46);
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle, K-major: rows of 128 bytes (64 bf16 along
+// K), 8-row groups 1024 bytes apart; within a 1024-byte-aligned group the 16-byte chunk j of row r
+// is stored at chunk j ^ r.  A K step of 16 elements advances the start address by 32 bytes.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+  return static_cast<uint64_t>((addr & 0x3FFFFu) >> 4) | (1ull << 16) | (static_cast<uint64_t>(1024 >> 4) << 32) |
+         (1ull << 46) | (2ull << 61);
 }
 
 // Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both K-major, N, M.
