@@ -646,8 +646,11 @@ def ours(args, w):
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic_from_profile(w.name),
                          "peak_kind": peak_kind, "algorithmic_bytes_per_launch": ideal,
-                         "kernel": kernel_name(w) + (f" + {backward_kernel_name(w)} (two launches per step)" if w.backward
-                                                     else " (one launch per step)")},
+                         "kernel": kernel_name(w) + (
+                             f" + the block backward ({block_bwd_launches} launches, the largest "
+                             f"{backward_kernel_name(w)})" if w.backward and w.block else
+                             f" + {backward_kernel_name(w)} (two launches per step)" if w.backward
+                             else " (one launch per step)")},
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": K * launches_per_step, "clocks": clocks}
     alu = alu_floor(w, torch.cuda.get_device_properties(dev).multi_processor_count, clocks.get("sm_mhz"))
     if alu["floor_us"] is not None:
