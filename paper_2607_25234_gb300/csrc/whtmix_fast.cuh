@@ -441,6 +441,25 @@ __device__ __forceinline__ void row_loc(long long b0, long long r, long long lv,
   *lim = static_cast<int>(n);
 }
 
+// Issued before pdl_wait(): asks L2 for the X rows [rb, re) of the first plane group that this
+// CTA's phase 1 reads, at most PREFETCH_BYTES of them, so that their HBM reads overlap the
+// previous kernel's tail.  A cache hint only: L2 is the point of coherence, so a line fetched
+// before the previous kernel's last writes to it still returns those writes.
+constexpr long long PREFETCH_BYTES = 128 * 1024;
+template <int D, int R, int Q>
+__device__ __forceinline__ void l2_prefetch_first_rows(const void* src, long long rb, long long re, long long lv) {
+  constexpr long long ES = D == DT_BF16 ? 2 : 4;
+  const long long r = rb + threadIdx.x;
+  if (r >= re || (r - rb) * (ES << R) >= PREFETCH_BYTES) return;
+  long long e0;
+  int lim;
+  row_loc<R, Q>(0, r, lv, &e0, &lim);
+  if (lim > 0)
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(src) + e0 * ES),
+                 "r"(static_cast<unsigned>(lim * ES))
+                 : "memory");
+}
+
 // ---------------------------------------------------------------------------------------------
 // Gains as phase 2 reads them, per column: storage position sp of a workspace row, whose element
 // j is logical plane element (j << R) + sigma_inv(sp).  at() is one element of the column, at2()
@@ -804,6 +823,10 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     __syncthreads();
     tmem_fence_after();
     tlane = tmem_slot + (static_cast<uint32_t>(32 * ((threadIdx.x >> 5) & 3)) << 16);
+  }
+  {
+    const long long rows = min(static_cast<long long>(P.gp), P.B) << Q;
+    l2_prefetch_first_rows<D, R, Q>(P.x, rows * blockIdx.x / gridDim.x, rows * (blockIdx.x + 1) / gridDim.x, P.lv);
   }
   // tensor memory is allocated before the wait: the previous kernel's CTA on this SM has left
   pdl_wait();
