@@ -89,6 +89,20 @@ typedef enum {
 WHTMIX_API int whtmix_forward(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
                    int dtype, void *stream);
 
+/* Forward mixer with a 16-bit exchange: the map of whtmix_forward (Section III-B, Eq. 1-4), same
+ * arguments, where only the storage between the three-phase kernel's phases differs.  Planes of
+ * 2^14 .. 2^23 elements that run the three-phase kernel (fp32 or bf16 I/O) keep their butterflies
+ * and the gain in fp32 but round the intermediate plane to bf16 (nearest, ties to even) at the
+ * two points where it crosses between SMs: after the row bits and after the column bits.  That
+ * halves the workspace traffic through L2.  Each rounding moves a value by at most 2^-9 of itself,
+ * so the output's relative L2 error grows by at most about 2^-9 (max|G| / min|G| + 1) over
+ * whtmix_forward's (the bf16 output rounding adds its own 2^-9); it is not bit-identical to
+ * whtmix_forward.  Every other shape (int32, planes held on chip, planes below 2^14 or above 2^23
+ * elements) runs exactly what whtmix_forward runs.  The paper has no such variant (it trains
+ * under bf16 autocast and states no kernel). */
+WHTMIX_API int whtmix_forward_x16(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
+                       int dtype, void *stream);
+
 /* Backward mixer: both gradients of the forward map.
  *   x      [B, N, C] the forward input              gains [N, C] G
  *   dy     [B, N, C] upstream gradient dL/dY          dx   [B, N, C] dL/dX (may equal dy)

@@ -16,7 +16,7 @@ INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libwhtmix.so")
 SOURCES = ["whtmix_capi.cu", "whtmix_fast_f32.cu", "whtmix_fast_bf16.cu", "whtmix_fast_sep_f32.cu", "whtmix_block.cu", "whtmix_plane.cu",
-           "whtmix_fast_sep_bf16.cu", "whtmix_noalloc.cu", "whtmix_proj.cu", "whtmix_block_bwd.cu"]
+           "whtmix_fast_sep_bf16.cu", "whtmix_fast_x16.cu", "whtmix_noalloc.cu", "whtmix_proj.cu", "whtmix_block_bwd.cu"]
 OBJDIR = os.path.join(LIBDIR, "obj")
 # the bench's memory-only floor model of the three-phase forward (bench.py --floor); not the mixer
 FLOOR_SOURCE = "bench_floor.cu"

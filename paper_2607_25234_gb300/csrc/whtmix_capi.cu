@@ -93,20 +93,21 @@ int check_shape(int64_t B, int64_t N, int64_t C, int dtype, int* m) {
   return WHTMIX_OK;
 }
 
-// Planes per group: as many as fit in `target` bytes of plane-group workspace (at least one).
-int planes_per_group(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES) {
+// Planes per group: as many as fit in `target` bytes of plane-group workspace (at least one);
+// `es` bytes per workspace element (2 for the bf16 exchange of whtmix_forward_x16).
+int planes_per_group(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES, size_t es = 4) {
   if (B == 0) return 1;
-  const size_t per = (size_t{1} << m) * 4 * (backward && m > TILE_BITS ? 2 : 1);
+  const size_t per = (size_t{1} << m) * es * (backward && m > TILE_BITS ? 2 : 1);
   int64_t gp = static_cast<int64_t>(target / per);
   if (gp < 1) gp = 1;
   if (gp > B) gp = B;
   return static_cast<int>(gp);
 }
 
-size_t workspace_bytes(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES) {
+size_t workspace_bytes(int64_t B, int m, int backward, size_t target = WS_TARGET_BYTES, size_t es = 4) {
   if (m <= TILE_BITS && !backward) return HEADER_BYTES;
-  const int gp = planes_per_group(B, m, backward, target);
-  const size_t per = (size_t{1} << m) * 4 * (backward && m > TILE_BITS ? 2 : 1);
+  const int gp = planes_per_group(B, m, backward, target, es);
+  const size_t per = (size_t{1} << m) * es * (backward && m > TILE_BITS ? 2 : 1);
   return HEADER_BYTES + per * static_cast<size_t>(gp);
 }
 
@@ -299,8 +300,9 @@ bool use_fast_backward(int dtype, int m) {
   return (dtype == WHTMIX_F32 || dtype == WHTMIX_BF16) && m >= 14 && m <= 23;
 }
 
+// ws16: the three-phase forward exchanges bf16 (whtmix_forward_x16); P.ws is then sized for it.
 template <int D>
-int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
+int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream, bool ws16 = false) {
   using A = typename Tr<D>::A;
   const int m = P.m;
   const size_t tile_bytes = sizeof(A) * TILE;
@@ -308,7 +310,8 @@ int dispatch(bool backward, const Params& P, int sms, cudaStream_t stream) {
   if (!backward) {
     if constexpr (D != DT_I32) {
       if (use_fast_forward(D, m)) {
-        const cudaError_t e = D == DT_BF16 ? fast::forward_bf16(P, sms, stream) : fast::forward_f32(P, sms, stream);
+        const cudaError_t e = ws16 ? (D == DT_BF16 ? fast::forward_x16_bf16(P, sms, stream) : fast::forward_x16_f32(P, sms, stream))
+                                   : (D == DT_BF16 ? fast::forward_bf16(P, sms, stream) : fast::forward_f32(P, sms, stream));
         return e == cudaSuccess ? WHTMIX_OK : cuda_fail(e);
       }
     }
@@ -459,7 +462,15 @@ struct Call {
   // scratch shared by every call: a wait that gave up in an earlier call must not leave counts
   // behind, and its error stays set until whtmix_sync reports it)
   bool reset_arrivals = false;
+  // whtmix_forward_x16: where the three-phase fast forward runs, it exchanges bf16 between its
+  // phases (every other kernel keeps its fp32 intermediate)
+  bool ws16 = false;
 };
+
+// The call runs the three-phase fast forward with the bf16 exchange workspace.
+bool x16_applies(const Call& c, int m) {
+  return c.ws16 && !c.backward && !c.separable && !c.w_in && use_fast_forward(c.dtype, m);
+}
 
 // Workspace layout of a call: the kernel workspace (barrier header + plane group) first, then
 // the separable tables or G / dG / partial sums, then the zero-padded copies.
@@ -479,7 +490,8 @@ Layout plan_call(const Call& c, int m) {
   const bool fast = c.backward ? use_fast_backward(c.dtype, m) : use_fast_forward(c.dtype, m);
   l.pad_copy = lv < L && !(fast && (lv * es) % 16 == 0);
   l.fast_sep = c.separable && !c.backward && !l.pad_copy && use_fast_separable(c.dtype, m, cbits);
-  l.base = workspace_bytes(c.B, m, c.backward, c.group_target);  // whtmix_workspace_bytes for a plain call
+  // whtmix_workspace_bytes for a plain call
+  l.base = workspace_bytes(c.B, m, c.backward, c.group_target, x16_applies(c, m) ? 2 : 4);
   size_t off = l.base;
   if (c.separable || l.pad_copy) off = align256(off);
   if (l.fast_sep) {
@@ -627,7 +639,8 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
   P.ws = wsb + HEADER_BYTES;
   P.B = c.B;
   P.m = m;
-  P.gp = planes_per_group(c.B, m, c.backward, c.group_target);
+  const bool ws16 = x16_applies(c, m);
+  P.gp = planes_per_group(c.B, m, c.backward, c.group_target, ws16 ? 2 : 4);
   P.scale = 1.0f / static_cast<float>(L);
   P.gt = c.gt;
   P.gc = c.gc;
@@ -670,8 +683,8 @@ int run(const Call& c, void* user_ws, size_t user_ws_bytes, bool use_user_ws, vo
     if (e != cudaSuccess) return cuda_fail(e);
   }
   switch (c.dtype) {
-    case WHTMIX_F32: rc = dispatch<DT_F32>(c.backward, P, sms, stream); break;
-    case WHTMIX_BF16: rc = dispatch<DT_BF16>(c.backward, P, sms, stream); break;
+    case WHTMIX_F32: rc = dispatch<DT_F32>(c.backward, P, sms, stream, ws16); break;
+    case WHTMIX_BF16: rc = dispatch<DT_BF16>(c.backward, P, sms, stream, ws16); break;
     default: rc = dispatch<DT_I32>(c.backward, P, sms, stream); break;
   }
   if (rc != WHTMIX_OK) return rc;
@@ -754,6 +767,13 @@ extern "C" {
 
 int whtmix_forward(const void* x, const void* gains, void* y, int64_t B, int64_t N, int64_t C, int dtype, void* stream) {
   return run(full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype), nullptr, 0, false, stream);
+}
+
+int whtmix_forward_x16(const void* x, const void* gains, void* y, int64_t B, int64_t N, int64_t C, int dtype,
+                       void* stream) {
+  Call c = full_call(false, x, gains, nullptr, y, nullptr, B, N, N, C, dtype);
+  c.ws16 = true;
+  return run(c, nullptr, 0, false, stream);
 }
 
 int whtmix_backward(const void* x, const void* gains, const void* dy, void* dx, void* dgains, int64_t B, int64_t N,

@@ -232,6 +232,45 @@ template <> struct IOv<DT_F32> {
 };
 
 // ---------------------------------------------------------------------------------------------
+// Workspace element: fp32 (the exact exchange), or bf16 for whtmix_forward_x16, where every value
+// that crosses between SMs is rounded to the nearest bf16 (ties to even) where it is written and
+// widened exactly where it is read; every butterfly and the gain stay fp32.  ld2/st2: elements
+// p[0], p[1] (p even).  The phase-3 staging holds a pair per slot (an fp32 pair, or one 32-bit
+// word of two bf16).
+struct WsF32 {
+  using T = float;
+  __device__ static __forceinline__ float ld(const float* p) { return __ldcg(p); }
+  __device__ static __forceinline__ void st(float* p, float v) { __stcg(p, v); }
+  __device__ static __forceinline__ float2 ld2(const float* p) { return __ldcg(reinterpret_cast<const float2*>(p)); }
+  __device__ static __forceinline__ void st2(float* p, float2 v) { __stcg(reinterpret_cast<float2*>(p), v); }
+  __device__ static __forceinline__ float2 staged(const float* stg, int slot) {
+    return *reinterpret_cast<const float2*>(stg + 2 * slot);
+  }
+};
+struct WsB16 {
+  using T = unsigned short;
+  __device__ static __forceinline__ float2 widen2(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+  }
+  __device__ static __forceinline__ float ld(const unsigned short* p) {
+    return __uint_as_float(static_cast<uint32_t>(__ldcg(p)) << 16);
+  }
+  __device__ static __forceinline__ void st(unsigned short* p, float v) {
+    __stcg(p, __bfloat16_as_ushort(__float2bfloat16_rn(v)));
+  }
+  __device__ static __forceinline__ float2 ld2(const unsigned short* p) {
+    return widen2(__ldcg(reinterpret_cast<const unsigned int*>(p)));
+  }
+  __device__ static __forceinline__ void st2(unsigned short* p, float2 v) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(v.x, v.y);
+    __stcg(reinterpret_cast<unsigned int*>(p), *reinterpret_cast<const unsigned int*>(&h));
+  }
+  __device__ static __forceinline__ float2 staged(const float* stg, int slot) {
+    return widen2(reinterpret_cast<const uint32_t*>(stg)[slot]);
+  }
+};
+
+// ---------------------------------------------------------------------------------------------
 // Asynchronous global -> shared copies (no registers held while in flight).
 __device__ __forceinline__ void cp_async16(float* smem_dst, const void* gsrc) {
   const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
@@ -293,11 +332,14 @@ __device__ __forceinline__ void stage_row_in(const void* src, long long e0, floa
 }
 // Phase 3 stages the first 32 of the 64 pairs each thread reads in layout P.
 __device__ __forceinline__ int pbase_of(int wt) { return 2 * (wt & 1) + 4 * ((wt >> 1) & 1) + 512 * (wt >> 2); }
-template <int R>
-__device__ __forceinline__ void stage_row_out(const float* src_ws, float* stg, int wt) {
+template <int R, class WS = WsF32>
+__device__ __forceinline__ void stage_row_out(const typename WS::T* src_ws, float* stg, int wt) {
   const int pbase = pbase_of(wt);
 #pragma unroll
-  for (int s = 0; s < 32; ++s) cp_async8(stg + (s * Row<R>::WORKER + wt) * 2, src_ws + sigma(pbase + 8 * s));
+  for (int s = 0; s < 32; ++s) {
+    if constexpr (sizeof(typename WS::T) == 4) cp_async8(stg + (s * Row<R>::WORKER + wt) * 2, src_ws + sigma(pbase + 8 * s));
+    else cp_async4(stg + s * Row<R>::WORKER + wt, reinterpret_cast<const float*>(src_ws + sigma(pbase + 8 * s)));
+  }
   cp_async_commit();
 }
 
@@ -330,8 +372,8 @@ __device__ __forceinline__ void round_v(float2 (&a)[16][4]) {
 // the next row's prefetch (element e0_next of src_next, lim_next of its elements stored, if
 // src_next is not null) is issued as soon as this row is in registers.  Elements of a row at
 // offsets >= lim are zero padding (never read).
-template <int D, int R>
-__device__ __forceinline__ void row_forward_in(const void* src, long long e0, int lim, float* dst_ws, float* xbuf,
+template <int D, int R, class WS = WsF32>
+__device__ __forceinline__ void row_forward_in(const void* src, long long e0, int lim, typename WS::T* dst_ws, float* xbuf,
                                                float* stg, int wt, int worker, const void* src_next, long long e0_next,
                                                int lim_next) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
@@ -385,27 +427,27 @@ __device__ __forceinline__ void row_forward_in(const void* src, long long e0, in
   bfly_all<64>(b);
   if constexpr (R == 14) bfly_lane4(b);
 #pragma unroll
-  for (int s = 0; s < 64; ++s) __stcg(reinterpret_cast<float2*>(dst_ws + sigma(pbase + 8 * s)), b[s]);
+  for (int s = 0; s < 64; ++s) WS::st2(dst_ws + sigma(pbase + 8 * s), b[s]);
 }
 
 // Phase 3 row: workspace (fp32) -> Y (dtype D), butterflies on all R row bits (mirror of phase 1).
 // The first half of the row's pairs arrives through the staging area; src_next (if not null) is
 // the next row, whose prefetch is issued once this row is in registers.
 // Only the row's first lim elements are stored (the rest is the cropped padding).
-template <int D, int R>
-__device__ __forceinline__ void row_forward_out(const float* src_ws, void* dst, long long e0, int lim, float* xbuf,
-                                                float* stg, int wt, int worker, const float* src_next) {
+template <int D, int R, class WS = WsF32>
+__device__ __forceinline__ void row_forward_out(const typename WS::T* src_ws, void* dst, long long e0, int lim, float* xbuf,
+                                                float* stg, int wt, int worker, const typename WS::T* src_next) {
   constexpr int WK = Row<R>::WORKER, VS = Row<R>::VSTRIDE;
   const int pbase = pbase_of(wt);
   float2 b[64];
 #pragma unroll
-  for (int s = 32; s < 64; ++s) b[s] = __ldcg(reinterpret_cast<const float2*>(src_ws + sigma(pbase + 8 * s)));
+  for (int s = 32; s < 64; ++s) b[s] = WS::ld2(src_ws + sigma(pbase + 8 * s));
   cp_async_wait_all();
 #pragma unroll
-  for (int s = 0; s < 32; ++s) b[s] = *reinterpret_cast<const float2*>(stg + (s * WK + wt) * 2);
+  for (int s = 0; s < 32; ++s) b[s] = WS::staged(stg, s * WK + wt);
   bfly_all<64>(b);  // round A: r3..r8 (and r9 for R = 14)
   if constexpr (R == 14) bfly_lane4(b);
-  if (src_next != nullptr) stage_row_out<R>(src_next, stg, wt);
+  if (src_next != nullptr) stage_row_out<R, WS>(src_next, stg, wt);
 #pragma unroll
   for (int s = 0; s < 64; ++s) *reinterpret_cast<float2*>(xbuf + xswz(pbase + 8 * s)) = b[s];
   worker_sync<R>(worker);
@@ -518,8 +560,9 @@ __device__ __forceinline__ long long sep_token_of(long long i, int cb) {
 // ---------------------------------------------------------------------------------------------
 // Phase 2, register variant (Q <= 6): a thread owns two adjacent storage positions (one logical
 // column pair) x 2^Q rows.
-template <int Q, int R, class GainT>
-__device__ __forceinline__ void col_pass_pairs(float* ws, const GainT& gain, float scale, int m, long long u_begin, long long u_end) {
+template <int Q, int R, class GainT, class WS = WsF32>
+__device__ __forceinline__ void col_pass_pairs(typename WS::T* ws, const GainT& gain, float scale, int m, long long u_begin,
+                                               long long u_end) {
   constexpr int NR = 1 << Q;
   const float2 sc = make_float2(scale, scale);
   for (long long u0 = u_begin; u0 < u_end; u0 += 2 * THREADS) {
@@ -527,34 +570,35 @@ __device__ __forceinline__ void col_pass_pairs(float* ws, const GainT& gain, flo
     if (u >= u_end) break;
     const long long b = u >> R;
     const int sp = static_cast<int>(u & ((1 << R) - 1));  // storage position (even); sp + 1 is column c + 1
-    float* base = ws + (b << m) + sp;
+    typename WS::T* base = ws + (b << m) + sp;
     const auto gc = gain.col(sp);
     float2 v[NR];
 #pragma unroll
-    for (int j = 0; j < NR; ++j) v[j] = __ldcg(reinterpret_cast<const float2*>(base + (static_cast<long long>(j) << R)));
+    for (int j = 0; j < NR; ++j) v[j] = WS::ld2(base + (static_cast<long long>(j) << R));
     bfly_all<NR>(v);
 #pragma unroll
     for (int j = 0; j < NR; ++j) v[j] = mul2(v[j], mul2(gain.at2(gc, j), sc));
     bfly_all<NR>(v);
 #pragma unroll
-    for (int j = 0; j < NR; ++j) __stcg(reinterpret_cast<float2*>(base + (static_cast<long long>(j) << R)), v[j]);
+    for (int j = 0; j < NR; ++j) WS::st2(base + (static_cast<long long>(j) << R), v[j]);
   }
 }
 
 // Phase 2, register variant for Q = 7: a thread owns one column of 128 rows as 64 pairs (j, j + 64).
-template <int R, class GainT>
-__device__ __forceinline__ void col_pass_single128(float* ws, const GainT& gain, float scale, int m, long long u_begin, long long u_end) {
+template <int R, class GainT, class WS = WsF32>
+__device__ __forceinline__ void col_pass_single128(typename WS::T* ws, const GainT& gain, float scale, int m, long long u_begin,
+                                                   long long u_end) {
   for (long long u0 = u_begin; u0 < u_end; u0 += THREADS) {
     const long long u = u0 + threadIdx.x;
     if (u >= u_end) break;
     const long long b = u >> R;
     const int sp = static_cast<int>(u & ((1 << R) - 1));
-    float* base = ws + (b << m) + sp;
+    typename WS::T* base = ws + (b << m) + sp;
     const auto gc = gain.col(sp);
     float2 v[64];
 #pragma unroll
     for (int j = 0; j < 64; ++j)
-      v[j] = make_float2(__ldcg(base + (static_cast<long long>(j) << R)), __ldcg(base + (static_cast<long long>(j + 64) << R)));
+      v[j] = make_float2(WS::ld(base + (static_cast<long long>(j) << R)), WS::ld(base + (static_cast<long long>(j + 64) << R)));
     bfly_all<64>(v);
 #pragma unroll
     for (int j = 0; j < 64; ++j) bf_in(v[j]);
@@ -570,8 +614,8 @@ __device__ __forceinline__ void col_pass_single128(float* ws, const GainT& gain,
     bfly_all<64>(v);
 #pragma unroll
     for (int j = 0; j < 64; ++j) {
-      __stcg(base + (static_cast<long long>(j) << R), v[j].x);
-      __stcg(base + (static_cast<long long>(j + 64) << R), v[j].y);
+      WS::st(base + (static_cast<long long>(j) << R), v[j].x);
+      WS::st(base + (static_cast<long long>(j + 64) << R), v[j].y);
     }
   }
 }
@@ -618,10 +662,11 @@ __device__ __forceinline__ void lane16_swap(float2 (&v)[8][W], int h) {
 // round C); MODE 2 is MODE 0 on the dY workspace, and at the gain step also reads the MODE 1
 // result at the same positions of xws, the transformed X column, and replaces it with the product
 // (W X)(W dY) times `scale` (the dG term of the plane).
-template <int Q, int R, class GainT, int MODE = 0>
-__device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, float scale, int m, long long u_begin,
+template <int Q, int R, class GainT, int MODE = 0, class WS = WsF32>
+__device__ __forceinline__ void col_pass_tmem(typename WS::T* ws, const GainT& gain, float scale, int m, long long u_begin,
                                               long long u_end, uint32_t tlane, float* xws = nullptr) {
   constexpr bool LANE_BIT = Q == 10;
+  static_assert(MODE == 0 || std::is_same<WS, WsF32>::value, "the backward modes: fp32 workspace");
   static_assert(MODE == 0 || (!LANE_BIT && !GainT::SEPARABLE), "the backward modes: Q = 8, 9, full gains");
   constexpr int ET_BITS = LANE_BIT ? 8 : Q - 1;        // 8, 7 for Q = 9, 8; 8 for Q = 10
   constexpr int ET = 1 << ET_BITS;
@@ -641,9 +686,9 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
     const long long uu = active ? u : u_begin;  // inactive lanes compute on a valid column, never store
     const long long b = uu >> R;
     const int sp = static_cast<int>(uu & ((1 << R) - 1));  // storage position of the column
-    float* colp = ws + (b << m) + sp;
+    typename WS::T* colp = ws + (b << m) + sp;
     const auto gcol = gain.col(sp);
-    float* own = colp + (static_cast<long long>(l4 * 2 * ET + hw * ET) << R);
+    typename WS::T* own = colp + (static_cast<long long>(l4 * 2 * ET + hw * ET) << R);
     // round A
 #pragma unroll 1
     for (int it = 0; it < ITA; ++it) {
@@ -651,7 +696,7 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 #pragma unroll
       for (int k = 0; k < 64; ++k) {
         const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
-        v[k] = make_float2(__ldcg(own + (k0 << R)), __ldcg(own + (k1 << R)));
+        v[k] = make_float2(WS::ld(own + (k0 << R)), WS::ld(own + (k1 << R)));
       }
       bfly_all<64>(v);
 #pragma unroll
@@ -788,8 +833,8 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 #pragma unroll
         for (int k = 0; k < 64; ++k) {
           const long long k0 = k + 64 * it, k1 = k0 + ET / 2;
-          __stcg(own + (k0 << R), v[k].x);
-          __stcg(own + (k1 << R), v[k].y);
+          WS::st(own + (k0 << R), v[k].x);
+          WS::st(own + (k1 << R), v[k].y);
         }
       }
     }
@@ -801,9 +846,11 @@ __device__ __forceinline__ void col_pass_tmem(float* ws, const GainT& gain, floa
 // ---------------------------------------------------------------------------------------------
 // Forward kernel: persistent grid (one CTA per SM, all resident), plane groups of P.gp planes,
 // three phases.  R and Q are template parameters so that every register array has a static size.
-template <int D, int R, int Q, bool SEP>
+// WS: the workspace element (WsF32, or WsB16 for whtmix_forward_x16; full gains only).
+template <int D, int R, int Q, bool SEP, class WS = WsF32>
 __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   static_assert((R == 13 && Q >= 1 && Q <= 10) || (R == 14 && (Q == 7 || Q == 9)), "supported row/column split");
+  static_assert(!SEP || std::is_same<WS, WsF32>::value, "separable gains: fp32 workspace (it holds the gain tables)");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int flag;
   __shared__ uint32_t tmem_slot;
@@ -813,7 +860,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
   const int worker = threadIdx.x / RW::WORKER, wt = threadIdx.x % RW::WORKER;
   float* xbuf = sm + worker * RW::LEN;
   float* stg = sm + SMEM_XBUF_BYTES / sizeof(float) + worker * RW::STAGE;
-  float* ws = static_cast<float*>(P.ws);
+  typename WS::T* ws = static_cast<typename WS::T*>(P.ws);
   const float* g = static_cast<const float*>(P.g);
   const int m = R + Q;
   uint32_t tlane = 0;
@@ -842,7 +889,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
     // phase 1: X -> ws, row bits (and, once, the separable gain tables exp(g_t), exp(g_c))
     if constexpr (SEP) {
       if (b0 == 0) {
-        float* tab = ws + (static_cast<long long>(P.gp) << m);
+        float* tab = reinterpret_cast<float*>(ws) + (static_cast<long long>(P.gp) << m);
         const long long n_t = 1ll << (m - P.cbits), n_tab = n_t + (1ll << P.cbits);
         for (long long i = static_cast<long long>(blockIdx.x) * THREADS + threadIdx.x; i < n_tab;
              i += static_cast<long long>(gridDim.x) * THREADS)
@@ -864,7 +911,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
       int lim, limn;
       row_loc<R, Q>(b0, r, P.lv, &e0, &lim);
       row_loc<R, Q>(b0, rn, P.lv, &e0n, &limn);
-      row_forward_in<D, R>(P.x, e0, lim, ws + (r << R), xbuf, stg, wt, worker, rn < re ? P.x : nullptr, e0n, limn);
+      row_forward_in<D, R, WS>(P.x, e0, lim, ws + (r << R), xbuf, stg, wt, worker, rn < re ? P.x : nullptr, e0n, limn);
     }
     if (!gsync()) break;
     // phase 2: column bits, gain, column bits
@@ -872,24 +919,24 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_fast(Params P) {
       using GainT = typename std::conditional<SEP, SepGain<R, Q>, FullGain<R>>::type;
       GainT gain;
       if constexpr (SEP) {
-        const float* tab = ws + (static_cast<long long>(P.gp) << m);
+        const float* tab = reinterpret_cast<const float*>(ws) + (static_cast<long long>(P.gp) << m);
         gain = GainT{tab, tab + (1ll << (m - P.cbits)), P.cbits};
       } else {
         gain = GainT{g};
       }
-      if constexpr (USE_TMEM) col_pass_tmem<Q, R>(ws, gain, P.scale, m, cb, ce, tlane);
-      else if constexpr (Q == 7) col_pass_single128<R>(ws, gain, P.scale, m, cb, ce);
-      else col_pass_pairs<Q, R>(ws, gain, P.scale, m, cb, ce);
+      if constexpr (USE_TMEM) col_pass_tmem<Q, R, GainT, 0, WS>(ws, gain, P.scale, m, cb, ce, tlane);
+      else if constexpr (Q == 7) col_pass_single128<R, GainT, WS>(ws, gain, P.scale, m, cb, ce);
+      else col_pass_pairs<Q, R, GainT, WS>(ws, gain, P.scale, m, cb, ce);
     }
     if (!gsync()) break;
     // phase 3: ws -> Y, row bits
-    if (rb + worker < re) stage_row_out<R>(ws + ((rb + worker) << R), stg, wt);
+    if (rb + worker < re) stage_row_out<R, WS>(ws + ((rb + worker) << R), stg, wt);
     for (long long r = rb + worker; r < re; r += RW::NWORKERS) {
       const long long rn = r + RW::NWORKERS;
       long long e0;
       int lim;
       row_loc<R, Q>(b0, r, P.lv, &e0, &lim);
-      row_forward_out<D, R>(ws + (r << R), P.y, e0, lim, xbuf, stg, wt, worker, rn < re ? ws + (rn << R) : nullptr);
+      row_forward_out<D, R, WS>(ws + (r << R), P.y, e0, lim, xbuf, stg, wt, worker, rn < re ? ws + (rn << R) : nullptr);
     }
     if (b0 + P.gp < P.B && !gsync()) break;
   }

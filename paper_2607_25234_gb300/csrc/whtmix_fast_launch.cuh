@@ -52,9 +52,9 @@ inline cudaError_t launch_persistent(const void* k, const Params& P, int sms, cu
   void* args[] = {&p};
   return launch_pdl(k, static_cast<unsigned>(sms), THREADS, smem, stream, args);
 }
-template <int D, int R, int Q, bool SEP>
+template <int D, int R, int Q, bool SEP, class WS = WsF32>
 cudaError_t launch_one(const Params& P, int sms, cudaStream_t stream) {
-  return launch_persistent(reinterpret_cast<const void*>(k_forward_fast<D, R, Q, SEP>), P, sms, stream);
+  return launch_persistent(reinterpret_cast<const void*>(k_forward_fast<D, R, Q, SEP, WS>), P, sms, stream);
 }
 template <int D, int R, int Q>
 cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
@@ -68,19 +68,20 @@ cudaError_t launch_bwd_one(const Params& P, int sms, cudaStream_t stream) {
 // per thread in registers, instead of 256-row columns in tensor memory: measured on sixteen such
 // planes (bf16), 138 us against 146 us per call.
 // SEP: separable log gains (P.gt, P.gc) instead of G; needs 1 <= P.cbits <= row bits.
-template <int D, bool SEP>
+// WS: the workspace element (WsB16: whtmix_forward_x16).
+template <int D, bool SEP, class WS = WsF32>
 cudaError_t launch_forward(const Params& P, int sms, cudaStream_t stream) {
   switch (P.m) {
-    case 14: return launch_one<D, 13, 1, SEP>(P, sms, stream);
-    case 15: return launch_one<D, 13, 2, SEP>(P, sms, stream);
-    case 16: return launch_one<D, 13, 3, SEP>(P, sms, stream);
-    case 17: return launch_one<D, 13, 4, SEP>(P, sms, stream);
-    case 18: return launch_one<D, 13, 5, SEP>(P, sms, stream);
-    case 19: return launch_one<D, 13, 6, SEP>(P, sms, stream);
-    case 20: return launch_one<D, 13, 7, SEP>(P, sms, stream);
-    case 21: return launch_one<D, 14, 7, SEP>(P, sms, stream);
-    case 22: return launch_one<D, 13, 9, SEP>(P, sms, stream);
-    case 23: return launch_one<D, 13, 10, SEP>(P, sms, stream);
+    case 14: return launch_one<D, 13, 1, SEP, WS>(P, sms, stream);
+    case 15: return launch_one<D, 13, 2, SEP, WS>(P, sms, stream);
+    case 16: return launch_one<D, 13, 3, SEP, WS>(P, sms, stream);
+    case 17: return launch_one<D, 13, 4, SEP, WS>(P, sms, stream);
+    case 18: return launch_one<D, 13, 5, SEP, WS>(P, sms, stream);
+    case 19: return launch_one<D, 13, 6, SEP, WS>(P, sms, stream);
+    case 20: return launch_one<D, 13, 7, SEP, WS>(P, sms, stream);
+    case 21: return launch_one<D, 14, 7, SEP, WS>(P, sms, stream);
+    case 22: return launch_one<D, 13, 9, SEP, WS>(P, sms, stream);
+    case 23: return launch_one<D, 13, 10, SEP, WS>(P, sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -112,6 +113,9 @@ cudaError_t forward_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t forward_bf16(const Params& P, int sms, cudaStream_t stream);
 cudaError_t backward_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t backward_bf16(const Params& P, int sms, cudaStream_t stream);
+// whtmix_fast_x16.cu: the forward with a bf16 exchange workspace
+cudaError_t forward_x16_f32(const Params& P, int sms, cudaStream_t stream);
+cudaError_t forward_x16_bf16(const Params& P, int sms, cudaStream_t stream);
 // whtmix_fast_sep_f32.cu / whtmix_fast_sep_bf16.cu
 cudaError_t forward_sep_f32(const Params& P, int sms, cudaStream_t stream);
 cudaError_t forward_sep_bf16(const Params& P, int sms, cudaStream_t stream);

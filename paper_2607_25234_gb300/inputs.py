@@ -95,6 +95,7 @@ class Workload:
     gains: str = "full"   # "full": G [N, C]; "separable": log gains g_t [N], g_c [C] (Eq. 2-3)
     padded_io: bool = False  # X, Y hold only the n_valid stored tokens; the library pads to N
     block: bool = False      # the whole block of Eq. 1-4: W_in projection, mixer, W_out projection
+    exchange: str = "f32"    # "bf16": whtmix_forward_x16, the intermediate plane exchanged in bf16
 
     @property
     def L(self) -> int:
@@ -150,6 +151,10 @@ WORKLOADS = {
     "block_train_fullimage_1x65536x128_bf16": Workload("block_train_fullimage_1x65536x128_bf16", 1, 65536, 128, "bf16",
                                                        backward=True, n_valid=2 * 135 * 240, block=True,
                                                        description="mixer block, training step: forward + backward"),
+    # the full-image forward with the 16-bit exchange between the three-phase kernel's phases
+    "fullimage_x16_1x65536x128_bf16": Workload("fullimage_x16_1x65536x128_bf16", 1, 65536, 128, "bf16",
+                                               n_valid=2 * 135 * 240, exchange="bf16",
+                                               description="full-image shape, forward, bf16 exchange workspace"),
     # the paper's mixer as trained: separable log gains and in-library padding
     "fullimage_paper_1x64800x128_bf16": Workload("fullimage_paper_1x64800x128_bf16", 1, 65536, 128, "bf16",
                                                  n_valid=2 * 135 * 240, padded_io=True, gains="separable",

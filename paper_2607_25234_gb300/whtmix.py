@@ -35,7 +35,7 @@ EXPORTS = ("whtmix_forward", "whtmix_backward", "whtmix_workspace_bytes", "whtmi
            "whtmix_backward_ex", "whtmix_sync", "whtmix_release_workspaces", "whtmix_status_string",
            "whtmix_last_cuda_error", "whtmix_plan", "whtmix_forward_noalloc", "whtmix_forward_separable",
            "whtmix_backward_separable", "whtmix_forward_padded", "whtmix_backward_padded", "whtmix_project",
-           "whtmix_block_forward", "whtmix_block_backward")
+           "whtmix_block_forward", "whtmix_block_backward", "whtmix_forward_x16")
 
 
 class WhtmixError(RuntimeError):
@@ -62,6 +62,7 @@ def library(path: str | None = None) -> ctypes.CDLL:
             lib.whtmix_backward.argtypes = [p, p, p, p, p, i64, i64, i64, i, p]
             lib.whtmix_forward_ex.argtypes = [p, p, p, i64, i64, i64, i, p, sz, p]
             lib.whtmix_forward_noalloc.argtypes = [p, p, p, i64, i64, i64, i, p]
+            lib.whtmix_forward_x16.argtypes = [p, p, p, i64, i64, i64, i, p]
             lib.whtmix_backward_ex.argtypes = [p, p, p, p, p, i64, i64, i64, i, p, sz, p]
             lib.whtmix_workspace_bytes.argtypes = [i64, i64, i64, i, i, ctypes.POINTER(sz)]
             lib.whtmix_sync.argtypes = [p]
@@ -148,6 +149,16 @@ def forward(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, s
     y = _out(out, x.shape, x.dtype, x.device, "out")
     _call("whtmix_forward", x.device, stream, library().whtmix_forward, x.data_ptr(), g.data_ptr(), y.data_ptr(),
           B, N, C, DTYPE_CODE[x.dtype])
+    return y
+
+
+def forward_x16(x: torch.Tensor, g: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """forward whose three-phase kernel rounds the exchanged intermediate plane to bf16 (half the
+    workspace traffic; butterflies and gain in fp32); other shapes run exactly as forward."""
+    B, N, C = _check_tensors(x, g)
+    y = _out(out, x.shape, x.dtype, x.device, "out")
+    _call("whtmix_forward_x16", x.device, stream, library().whtmix_forward_x16, x.data_ptr(), g.data_ptr(),
+          y.data_ptr(), B, N, C, DTYPE_CODE[x.dtype])
     return y
 
 
