@@ -39,6 +39,10 @@ int main(void) {
   EXPECT(whtmix_forward(x, g, P(base + 16), 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_ALIAS);
   EXPECT(whtmix_forward(x, g, g, 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_ALIAS);
   EXPECT(whtmix_forward(NULL, NULL, NULL, 0, 4, 4, WHTMIX_BF16, NULL), WHTMIX_OK); /* empty batch */
+  EXPECT(whtmix_forward_x16(NULL, g, y, 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_INVALID_ARG);
+  EXPECT(whtmix_forward_x16(x, g, y, 1, 6, 4, WHTMIX_BF16, NULL), WHTMIX_ERR_BAD_SHAPE);
+  EXPECT(whtmix_forward_x16(x, g, P(base + 16), 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_ALIAS);
+  EXPECT(whtmix_forward_x16(NULL, NULL, NULL, 0, 4, 4, WHTMIX_BF16, NULL), WHTMIX_OK);
 
   /* backward */
   EXPECT(whtmix_backward(x, g, dy, dx, NULL, 1, 4, 4, WHTMIX_F32, NULL), WHTMIX_ERR_INVALID_ARG);

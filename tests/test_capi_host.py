@@ -293,3 +293,19 @@ def test_pad_tokens_helper():
     for bad in (4, 12):
         with pytest.raises(ValueError):
             whtmix.pad_tokens(x, bad)
+
+
+def xfwd(lib, x=FAKE, g=2 * FAKE, y=3 * FAKE, B=1, N=4, C=4, dtype=0):
+    return lib.whtmix_forward_x16(x, g, y, B, N, C, dtype, None)
+
+
+def test_x16_checks_its_arguments_as_the_forward_does(lib):
+    # whtmix_forward_x16 goes through the forward's host checks: the same status for every case
+    cases = [dict(x=None), dict(g=None), dict(y=None), dict(B=-1), dict(N=0), dict(N=6), dict(C=12),
+             dict(N=1 << 24, C=1 << 7), dict(B=(1 << 56) + 1), dict(dtype=3), dict(x=FAKE + 4),
+             dict(y=3 * FAKE + 8), dict(y=FAKE + 16), dict(y=2 * FAKE), dict(B=0),
+             dict(x=None, g=None, y=None, B=0)]
+    for kw in cases:
+        assert xfwd(lib, **kw) == fwd(lib, **kw), kw
+    passes_every_check(lambda: xfwd(lib, y=FAKE))                     # exact in place
+    passes_every_check(lambda: xfwd(lib, N=65536, C=128, dtype=1, x=FAKE, g=(1 << 40), y=(1 << 41)))
