@@ -46,7 +46,6 @@ KERNEL_FAMILY_SOURCES = {
     "k_backward_fast": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_fast_launch.cuh", "whtmix_fast_bwd.cuh"),
     "k_block_fast": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_block.cuh", "whtmix_block.cu"),
     "k_forward_plane": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_plane.cuh", "whtmix_plane.cu"),
-    "k_forward_row1": ("whtmix_kernels.cuh", "whtmix_fast.cuh", "whtmix_plane.cuh", "whtmix_plane.cu"),
 }
 
 
@@ -64,8 +63,6 @@ def kernel_name(w) -> str:
     padded_ok = w.n_valid is None or (w.n_valid * w.C * (2 if w.dtype == "bf16" else 4)) % 16 == 0
     if (w.dtype in ("f32", "bf16") and 14 <= m <= 16 and (m < 16 or w.B >= 80) and w.gains == "full"
             and not w.block and (not w.padded_io or padded_ok)):
-        if m == 14:
-            return f"k_forward_row1<{w.dtype}> (one plane per worker of 128 threads, in registers)"
         return f"k_forward_plane<{w.dtype}, column bits {m - 14}> (one plane per CTA, in tensor memory)"
     if w.dtype in ("f32", "bf16") and 14 <= m <= 23:
         r = 14 if m == 21 else 13

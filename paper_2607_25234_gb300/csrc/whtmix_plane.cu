@@ -11,7 +11,7 @@ namespace whtmix {
 namespace pln {
 
 // Per device and kernel: raise the dynamic shared memory limit once.
-inline cudaError_t prepare(const void* k, size_t smem = SMEM_BYTES) {
+inline cudaError_t prepare(const void* k) {
   static std::mutex mu;
   static std::map<std::pair<int, const void*>, cudaError_t> done;
   int dev = 0;
@@ -20,7 +20,7 @@ inline cudaError_t prepare(const void* k, size_t smem = SMEM_BYTES) {
   std::lock_guard<std::mutex> lk(mu);
   auto it = done.find({dev, k});
   if (it != done.end()) return it->second;
-  e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(SMEM_BYTES));
   done[{dev, k}] = e;
   return e;
 }
@@ -35,21 +35,10 @@ cudaError_t launch_cb(const Params& P, cudaStream_t stream) {
   return launch_pdl(k, static_cast<unsigned>(P.B), THREADS, SMEM_BYTES, stream, args);
 }
 
-// One-row planes (2^14 elements): one worker of 128 threads per plane, two planes per SM.
-template <int D>
-cudaError_t launch_row1(const Params& P, cudaStream_t stream) {
-  const void* k = reinterpret_cast<const void*>(k_forward_row1<D>);
-  cudaError_t e = prepare(k, ROW1_SMEM_BYTES);
-  if (e != cudaSuccess) return e;
-  Params p = P;
-  void* args[] = {&p};
-  return launch_pdl(k, static_cast<unsigned>(P.B), WK, ROW1_SMEM_BYTES, stream, args);
-}
-
 template <int D>
 cudaError_t launch(const Params& P, cudaStream_t stream) {
   switch (P.m) {
-    case 14: return launch_row1<D>(P, stream);
+    case 14: return launch_cb<D, 0>(P, stream);
     case 15: return launch_cb<D, 1>(P, stream);
     case 16: return launch_cb<D, 2>(P, stream);
     default: return cudaErrorInvalidValue;

@@ -79,9 +79,8 @@ __device__ __forceinline__ void pairs_from_tmem(uint32_t ta, float2 (&b)[64]) {
 // next row (src_next, if not null) is staged behind it.  Each thread reads back only the chunks it
 // copied, so the staging area needs no barrier.
 template <int D>
-__device__ __forceinline__ void row_in_regs(const void* src, long long e0, int lim, float* buf, float* stg, int wt,
-                                            int worker, const void* src_next, long long e0_next, int lim_next,
-                                            float2 (&b)[64]) {
+__device__ __forceinline__ void row_in(const void* src, long long e0, int lim, float* buf, float* stg, int wt,
+                                       int worker, uint32_t ta, const void* src_next, long long e0_next, int lim_next) {
   constexpr int VS = ROW / 16;
   float2 a[16][4];
   if constexpr (D == DT_F32) {
@@ -123,6 +122,7 @@ __device__ __forceinline__ void row_in_regs(const void* src, long long e0, int l
     }
   fast::worker_sync<R>(worker);
   const int pbase = fast::pbase_of(wt);
+  float2 b[64];
 #pragma unroll
   for (int s = 0; s < 64; ++s) b[s] = *reinterpret_cast<const float2*>(buf + fast::xswz(pbase + 8 * s));
   fast::worker_sync<R>(worker);  // the buffer is free for the worker's next row
@@ -130,22 +130,17 @@ __device__ __forceinline__ void row_in_regs(const void* src, long long e0, int l
   for (int s = 0; s < 64; ++s) fast::bf_in(b[s]);
   fast::bfly_all<64>(b);
   fast::bfly_lane4(b);
-}
-template <int D>
-__device__ __forceinline__ void row_in(const void* src, long long e0, int lim, float* buf, float* stg, int wt,
-                                       int worker, uint32_t ta, const void* src_next, long long e0_next, int lim_next) {
-  float2 b[64];
-  row_in_regs<D>(src, e0, lim, buf, stg, wt, worker, src_next, e0_next, lim_next, b);
   pairs_to_tmem(ta, b);
 }
 
 // Phase 3 row: this thread's pairs from TMEM at ta -> the 14 row bits -> Y (elements e0 ..., only
 // the first lim stored).
 template <int D>
-__device__ __forceinline__ void row_out_regs(float2 (&b)[64], float* buf, void* dst, long long e0, int lim, int wt,
-                                             int worker) {
+__device__ __forceinline__ void row_out(uint32_t ta, float* buf, void* dst, long long e0, int lim, int wt, int worker) {
   constexpr int VS = ROW / 16;
   const int pbase = fast::pbase_of(wt);
+  float2 b[64];
+  pairs_from_tmem(ta, b);
   fast::bfly_all<64>(b);
   fast::bfly_lane4(b);
 #pragma unroll
@@ -168,12 +163,6 @@ __device__ __forceinline__ void row_out_regs(float2 (&b)[64], float* buf, void* 
   fast::round_v(a);
 #pragma unroll
   for (int v = 0; v < 16; ++v) fast::IOv<D>::st8_lim(dst, e0 + 8 * wt + VS * v, a[v], lim - (8 * wt + VS * v));
-}
-template <int D>
-__device__ __forceinline__ void row_out(uint32_t ta, float* buf, void* dst, long long e0, int lim, int wt, int worker) {
-  float2 b[64];
-  pairs_from_tmem(ta, b);
-  row_out_regs<D>(b, buf, dst, e0, lim, wt, worker);
 }
 
 // Phase 2: pairs [32 worker, 32 worker + 32) of this lane's 64 positions, in two chunks of 16,
@@ -285,38 +274,6 @@ __global__ void __launch_bounds__(THREADS, 1) k_forward_plane(Params P) {
   __syncthreads();
   fast::tmem_fence_after();
   if (threadIdx.x < 32) fast::tmem_dealloc_512(tmem_slot);
-}
-
-// Planes of one row (2^14 elements): the transform is the row bits, the gain and the row bits
-// again, so one worker of 128 threads keeps the plane in registers from X to Y -- no tensor
-// memory and no CTA-wide barrier.  96 KiB of shared memory (an exchange buffer and a staging
-// area), so two CTAs share an SM.
-constexpr size_t ROW1_SMEM_BYTES = (ROW + STG) * sizeof(float);
-template <int D>
-__global__ void __launch_bounds__(WK, 2) k_forward_row1(Params P) {
-  extern __shared__ __align__(16) float r1_smem[];
-  const long long b = blockIdx.x;
-  const int wt = threadIdx.x;
-  float* buf = r1_smem;
-  float* stg = r1_smem + ROW;
-  pdl_wait();
-  long long e0;
-  int lim;
-  fast::row_loc<R, 0>(0, b, P.lv, &e0, &lim);
-  fast::stage_row_in<D, R>(P.x, e0, stg, wt, lim);
-  float2 v[64];
-  row_in_regs<D>(P.x, e0, lim, buf, stg, wt, 0, nullptr, 0, 0, v);
-  // the gain G/L at this thread's row positions pbase + 8 s, + 1
-  const int pbase = fast::pbase_of(wt);
-  const float2 sc = make_float2(P.scale, P.scale);
-  const float* g = static_cast<const float*>(P.g);
-#pragma unroll
-  for (int s = 0; s < 64; ++s) {
-    const float2 gg = __ldg(reinterpret_cast<const float2*>(g + pbase + 8 * s));
-    v[s] = fast::mul2(v[s], fast::mul2(gg, sc));
-  }
-  row_out_regs<D>(v, buf, P.y, e0, lim, wt, 0);
-  pdl_trigger();
 }
 
 }  // namespace pln

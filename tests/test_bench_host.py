@@ -32,7 +32,7 @@ def test_kernel_each_workload_launches():
     assert bench.kernel_name(W["fullimage_1x65536x128_bf16"]) == "k_forward_fast<bf16, R=13, Q=10>"
     assert bench.kernel_name(W["longseq_32x4096x64_f32"]) == "k_forward_fast<f32, R=13, Q=5>"
     assert bench.kernel_name(W["epipolar_128x512x128_bf16"]).startswith("k_forward_plane<bf16, column bits 2>")
-    assert bench.kernel_name(W["tiny_1x256x64_f32"]).startswith("k_forward_row1<f32>")
+    assert bench.kernel_name(W["tiny_1x256x64_f32"]).startswith("k_forward_plane<f32, column bits 0>")
     assert bench.kernel_name(W["train_16x8192x256_bf16"]) == "k_forward_fast<bf16, R=14, Q=7>"
     assert bench.backward_kernel_name(W["train_16x8192x256_bf16"]) == "k_backward_fast<bf16, R=14, Q=7>"
     assert bench.backward_kernel_name(W["fullimage_train_1x65536x128_bf16"]) == "k_backward_fast<bf16, R=14, Q=9>"
