@@ -117,3 +117,14 @@ def test_reference_arm_line_matches_ours_in_config_and_metric(monkeypatch, capsy
         assert line["impl"] == "reference" and line["metric"] == metric
         assert line["config"] == bench.workload_config(small, 1, bench.device_l2_bytes())
         assert line["cpu_baseline"]["cores"] >= 1 and line["value"] > 0
+
+
+def test_bf16_exchange_workload():
+    # the same shape, bytes and kernel as the full-image workload, with the exchange marked
+    w, ref = W["fullimage_x16_1x65536x128_bf16"], W["fullimage_1x65536x128_bf16"]
+    assert w.ideal_bytes() == ref.ideal_bytes() == 67_108_864
+    assert bench.kernel_name(w) == "k_forward_fast<bf16, R=13, Q=10, bf16 exchange>"
+    cfg, cfg_ref = bench.workload_config(w, 1, 126 << 20), bench.workload_config(ref, 1, 126 << 20)
+    assert cfg["exchange"] == "bf16" and cfg_ref["exchange"] == "f32"
+    assert {k: v for k, v in cfg.items() if k not in ("workload", "exchange")} == \
+        {k: v for k, v in cfg_ref.items() if k not in ("workload", "exchange")}
