@@ -97,9 +97,9 @@ WHTMIX_API int whtmix_forward(const void *x, const void *gains, void *y, int64_t
  * halves the workspace traffic through L2.  Each rounding moves a value by at most 2^-8 of itself,
  * so the output's relative L2 error grows by at most 2^-8 (max|G| / min|G| + 1) over
  * whtmix_forward's (measured: 2.3e-3 with fp32 I/O, 2.9e-3 with bf16 I/O, gains near 1); it is
- * not bit-identical to whtmix_forward.  Every other shape (int32, planes held on chip, planes below 2^14 or above 2^23
- * elements) runs exactly what whtmix_forward runs.  The paper has no such variant (it trains
- * under bf16 autocast and states no kernel). */
+ * not bit-identical to whtmix_forward.  Every other shape (int32, planes held on chip, planes
+ * below 2^14 or above 2^23 elements) runs exactly what whtmix_forward runs.  The paper has no
+ * such variant (it trains under bf16 autocast and states no kernel). */
 WHTMIX_API int whtmix_forward_x16(const void *x, const void *gains, void *y, int64_t B, int64_t N, int64_t C,
                        int dtype, void *stream);
 
